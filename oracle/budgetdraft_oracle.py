@@ -1,0 +1,314 @@
+"""Plain fp64 CPU oracle for the KV-cache attention of one BudgetDraft speculative step.
+
+TEST INFRASTRUCTURE ONLY.  Nothing on the product path may import or call this
+module: only the test suite, ``__graft_entry__.smoke()`` and the CPU-baseline leg
+of ``bench.py`` use it.  It shares no code with the CUDA path.
+
+Every function is the plain definition of what the step computes, written with
+numpy in float64.  Inputs are the bf16 values the kernels see, widened exactly to
+float64 by the caller.  Nothing here is blocked, fused or reordered: a reader
+can check each function against the paper by eye.
+
+Paper references (BudgetDraft, arXiv 2606.00144):
+  * Sparse drafter view K_S^sp(B) selected from the drafter prefix cache under a
+    KV budget B: Sec. 3.1 (Eq. p_S) and the TopKChunks construction in Sec. 3.4
+    ("partition the prefix cache into chunks, score each chunk by cumulative
+    attention weight, keep the top floor(B/s) chunks"), used by Algorithm 1
+    step 4 and by the sparsify line of Algorithm 2.
+  * Draft step: gamma autoregressive drafter steps over K_S^sp(B) (Algorithm 2,
+    Draft; Sec. 3.5).
+  * Verify step: the verifier checks all gamma drafts in one forward over the
+    full cache K_L^full (Algorithm 2, Verify; Sec. 3.5).
+  * Cache update: accepted tokens are appended to both caches (Algorithm 2,
+    Update), which is why the drafter's own new rows join its sparse view.
+
+Readings where the paper is silent (each is listed in the design doc):
+  * softmax scale 1/sqrt(d), no soft-cap; caches hold post-RoPE keys, so a row
+    gathered by index keeps its position (Sec. 3.4, explicit position IDs);
+  * "cumulative attention weight" of key k = sum over the GQA group's heads and
+    over a window of the last W context queries of their causal softmax
+    probability on k (token level, s = 1, with sink and recent positions always
+    kept, as the graded workloads specify); ties at the budget boundary go to
+    the lower position; the kept set is returned in ascending order;
+  * chunk level (s > 1): chunks are aligned at multiples of s from position 0,
+    a chunk's score is the sum of its middle members' scores, ties go to the
+    lower chunk; the sink/recent rule is the same;
+  * query i of a verify block sits at position t_ctx + i and sees keys
+    [0, t_ctx + i]; draft pass j sees the selected rows plus its own rows
+    t_ctx .. t_ctx + j.
+"""
+
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+NEG_INF = float("-inf")
+
+
+# ---------------------------------------------------------------------------
+# Attention by definition (Sec. 3.1: the drafter's p_S over K_S^sp(B) and the
+# verifier's p_L over K_L^full are both ordinary softmax attention).
+# ---------------------------------------------------------------------------
+
+def attention(q: np.ndarray, keys: np.ndarray, values: np.ndarray, scale: float):
+    """Softmax attention of one query over a set of key/value rows.
+
+    q: [d]; keys, values: [m, d] (float64).  Returns (o [d], lse) with
+        s_k = scale * (q . k_k),  lse = log sum_k exp(s_k),
+        o = sum_k exp(s_k - lse) v_k.
+    An empty key set gives o = 0 and lse = -inf (the neutral element of the
+    log-sum-exp merge below).
+    """
+    q = np.asarray(q, dtype=np.float64)
+    keys = np.asarray(keys, dtype=np.float64)
+    values = np.asarray(values, dtype=np.float64)
+    if keys.shape[0] == 0:
+        return np.zeros(values.shape[1], dtype=np.float64), NEG_INF
+    s = scale * (keys @ q)
+    m = s.max()
+    e = np.exp(s - m)
+    l = e.sum()
+    o = (e @ values) / l
+    return o, m + math.log(l)
+
+
+def combine(o_part: np.ndarray, lse_part: np.ndarray):
+    """Merge attention results computed over disjoint key sets.
+
+    o_part: [n, rows, d], each row normalised over its own key set;
+    lse_part: [n, rows].  With L = log sum_s exp(lse_s), the merged row is
+    sum_s exp(lse_s - L) o_s, which equals attention over the union of the key
+    sets.  Rows whose parts are all empty give o = 0, L = -inf.
+    """
+    o_part = np.asarray(o_part, dtype=np.float64)
+    lse_part = np.asarray(lse_part, dtype=np.float64)
+    n, rows, d = o_part.shape
+    o = np.zeros((rows, d), dtype=np.float64)
+    lse = np.full(rows, NEG_INF, dtype=np.float64)
+    for r in range(rows):
+        finite = np.isfinite(lse_part[:, r])
+        if not finite.any():
+            continue
+        m = lse_part[finite, r].max()
+        w = np.exp(lse_part[finite, r] - m)
+        L = m + math.log(w.sum())
+        lse[r] = L
+        o[r] = (np.exp(lse_part[finite, r] - L)[:, None] * o_part[finite, r, :]).sum(axis=0)
+    return o, lse
+
+
+# ---------------------------------------------------------------------------
+# Verify step (Algorithm 2, Verify): n_q = gamma + 1 queries over the full cache
+# with a causal mask inside the block.
+# ---------------------------------------------------------------------------
+
+def verify_attn(q: np.ndarray, k_cache: np.ndarray, v_cache: np.ndarray, t_ctx: int):
+    """q: [b, h_q, n_q, d]; caches: [b, h_kv, t_cap, d].
+
+    Query i of head h sits at position t_ctx + i and attends to keys
+    [0, t_ctx + i] of KV head h // (h_q / h_kv).  Returns o [b, h_q, n_q, d]
+    and lse [b, h_q, n_q].
+    """
+    b, h_q, n_q, d = q.shape
+    h_kv = k_cache.shape[1]
+    group = h_q // h_kv
+    scale = 1.0 / math.sqrt(d)
+    o = np.zeros((b, h_q, n_q, d), dtype=np.float64)
+    lse = np.zeros((b, h_q, n_q), dtype=np.float64)
+    for bi in range(b):
+        for h in range(h_q):
+            kv = h // group
+            for i in range(n_q):
+                last = t_ctx + i
+                o[bi, h, i], lse[bi, h, i] = attention(
+                    q[bi, h, i], k_cache[bi, kv, : last + 1], v_cache[bi, kv, : last + 1], scale)
+    return o, lse
+
+
+# ---------------------------------------------------------------------------
+# Draft step (Algorithm 2, Draft): pass j of the gamma drafter passes, one query
+# per head over the sparse view plus the drafter's own new rows.
+# ---------------------------------------------------------------------------
+
+def draft_attn(q: np.ndarray, k_cache: np.ndarray, v_cache: np.ndarray,
+               idx: np.ndarray, count: np.ndarray, t_ctx: int, step_j: int):
+    """q: [b, h_q, d]; idx: [b, h_kv, budget] (positions); count: [b, h_kv].
+
+    Pass j attends to rows idx[b, kv, :count[b, kv]] together with rows
+    t_ctx .. t_ctx + step_j (the tokens drafted so far, own row included).
+    Returns o [b, h_q, d], lse [b, h_q].
+    """
+    b, h_q, d = q.shape
+    h_kv = k_cache.shape[1]
+    group = h_q // h_kv
+    scale = 1.0 / math.sqrt(d)
+    o = np.zeros((b, h_q, d), dtype=np.float64)
+    lse = np.zeros((b, h_q), dtype=np.float64)
+    for bi in range(b):
+        for h in range(h_q):
+            kv = h // group
+            rows = list(idx[bi, kv, : int(count[bi, kv])]) + list(range(t_ctx, t_ctx + step_j + 1))
+            rows = np.asarray(rows, dtype=np.int64)
+            o[bi, h], lse[bi, h] = attention(q[bi, h], k_cache[bi, kv, rows], v_cache[bi, kv, rows], scale)
+    return o, lse
+
+
+# ---------------------------------------------------------------------------
+# Budget selection (Sec. 3.4 TopKChunks; Algorithm 2, sparsify).
+# ---------------------------------------------------------------------------
+
+def window_positions(t_ctx: int, window: int) -> np.ndarray:
+    """Positions of the observation window: the last W context positions."""
+    return np.arange(t_ctx - window, t_ctx, dtype=np.int64)
+
+
+def window_lse(q_win: np.ndarray, k_cache: np.ndarray, t_ctx: int):
+    """Softmax normaliser of each window query over its causal prefix.
+
+    q_win: [b, h_q, W, d]; window row w sits at p_w = t_ctx - W + w and
+    attends to keys [0, p_w].  Returns lse [b, h_q, W].
+    """
+    b, h_q, window, d = q_win.shape
+    h_kv = k_cache.shape[1]
+    group = h_q // h_kv
+    scale = 1.0 / math.sqrt(d)
+    pos = window_positions(t_ctx, window)
+    lse = np.zeros((b, h_q, window), dtype=np.float64)
+    for bi in range(b):
+        for h in range(h_q):
+            kv = h // group
+            for w in range(window):
+                s = scale * (k_cache[bi, kv, : pos[w] + 1] @ q_win[bi, h, w])
+                m = s.max()
+                lse[bi, h, w] = m + math.log(np.exp(s - m).sum())
+    return lse
+
+
+def window_scores(q_win: np.ndarray, k_cache: np.ndarray, lse_win: np.ndarray, t_ctx: int):
+    """Cumulative attention weight of every context key, pooled over the group.
+
+    score[b, kv, k] = sum over heads h of group kv and window rows w with
+    k <= p_w of exp(scale * q_{h,w} . k_k - lse_{h,w}), i.e. the sum of the
+    window rows' softmax probabilities on key k.  Returns [b, h_kv, t_ctx].
+    """
+    b, h_q, window, d = q_win.shape
+    h_kv = k_cache.shape[1]
+    group = h_q // h_kv
+    scale = 1.0 / math.sqrt(d)
+    pos = window_positions(t_ctx, window)
+    score = np.zeros((b, h_kv, t_ctx), dtype=np.float64)
+    for bi in range(b):
+        for kv in range(h_kv):
+            keys = k_cache[bi, kv, :t_ctx]
+            for g in range(group):
+                h = kv * group + g
+                for w in range(window):
+                    p = np.exp(scale * (keys @ q_win[bi, h, w]) - lse_win[bi, h, w])
+                    p[pos[w] + 1:] = 0.0          # causal: row w sees [0, p_w]
+                    score[bi, kv] += p
+    return score
+
+
+def topk_lower_index(values: np.ndarray, labels: np.ndarray, k: int) -> np.ndarray:
+    """The k labels with the largest values; equal values prefer the lower label."""
+    order = np.lexsort((labels, -values))        # primary: value desc, then label asc
+    return labels[order[:k]]
+
+
+def select_from_scores(score: np.ndarray, t_ctx: int, budget: int, n_sink: int,
+                       n_recent: int, chunk: int = 1) -> np.ndarray:
+    """Kept positions of one (sequence, KV head), ascending.
+
+    score: [t_ctx] cumulative attention weights.  If budget >= t_ctx every
+    position is kept.  Otherwise keep the sinks [0, n_sink), the recent
+    positions [t_ctx - n_recent, t_ctx) and, from the middle
+    [n_sink, t_ctx - n_recent):
+      * chunk == 1: the top (budget - n_sink - n_recent) positions by score;
+      * chunk == s > 1: the top floor((budget - n_sink - n_recent) / s) chunks
+        (chunk c covers positions [c s, c s + s) intersected with the middle),
+        a chunk scored by the sum of its members' scores.
+    Ties go to the lower position (lower chunk).
+    """
+    if budget >= t_ctx:
+        return np.arange(t_ctx, dtype=np.int64)
+    lo, hi = n_sink, t_ctx - n_recent
+    mid = np.arange(lo, hi, dtype=np.int64)
+    free = budget - n_sink - n_recent
+    if chunk == 1:
+        chosen = topk_lower_index(score[lo:hi], mid, free)
+    else:
+        first, last = lo // chunk, (hi - 1) // chunk
+        chunk_ids = np.arange(first, last + 1, dtype=np.int64)
+        chunk_score = np.array([score[max(c * chunk, lo): min(c * chunk + chunk, hi)].sum()
+                                for c in chunk_ids])
+        top = topk_lower_index(chunk_score, chunk_ids, free // chunk)
+        chosen = np.concatenate([np.arange(max(c * chunk, lo), min(c * chunk + chunk, hi))
+                                 for c in top] + [np.zeros(0, dtype=np.int64)])
+    keep = np.concatenate([np.arange(0, lo), chosen, np.arange(hi, t_ctx)]).astype(np.int64)
+    return np.sort(keep)
+
+
+def select_budget(q_win: np.ndarray, k_cache: np.ndarray, t_ctx: int, budget: int,
+                  n_sink: int, n_recent: int, chunk: int = 1, lse_win: np.ndarray | None = None):
+    """Sparse drafter view K_S^sp(B) of every (sequence, KV head).
+
+    Returns (idx [b, h_kv, budget] int64 padded with -1, count [b, h_kv],
+    score [b, h_kv, t_ctx]).  lse_win defaults to the oracle's own window_lse.
+    """
+    b, h_q, window, d = q_win.shape
+    h_kv = k_cache.shape[1]
+    if lse_win is None:
+        lse_win = window_lse(q_win, k_cache, t_ctx)
+    score = window_scores(q_win, k_cache, lse_win, t_ctx)
+    idx = np.full((b, h_kv, budget), -1, dtype=np.int64)
+    count = np.zeros((b, h_kv), dtype=np.int64)
+    for bi in range(b):
+        for kv in range(h_kv):
+            keep = select_from_scores(score[bi, kv], t_ctx, budget, n_sink, n_recent, chunk)
+            idx[bi, kv, : keep.size] = keep
+            count[bi, kv] = keep.size
+    return idx, count, score
+
+
+def boundary_score(score_row: np.ndarray, t_ctx: int, budget: int, n_sink: int, n_recent: int):
+    """Score of the last middle position admitted at token level (the B-th boundary).
+
+    Returns None when nothing is ranked (budget >= t_ctx or no free slot).
+    """
+    free = budget - n_sink - n_recent
+    if budget >= t_ctx or free <= 0:
+        return None
+    mid = np.sort(score_row[n_sink: t_ctx - n_recent])[::-1]
+    return float(mid[free - 1])
+
+
+# ---------------------------------------------------------------------------
+# One speculative step (Algorithm 2: sparsify, Draft x gamma, Verify).
+# ---------------------------------------------------------------------------
+
+def spec_step(k_cache, v_cache, q_win, q_draft, q_verify, t_ctx, budget, n_sink, n_recent,
+              lse_win=None, chunk=1):
+    """q_draft: [gamma, b, h_q, d]; q_verify: [b, h_q, gamma + 1, d].
+
+    Returns a dict with idx, count, score, draft_o [gamma, b, h_q, d],
+    draft_lse [gamma, b, h_q], verify_o, verify_lse.
+    """
+    idx, count, score = select_budget(q_win, k_cache, t_ctx, budget, n_sink, n_recent,
+                                      chunk, lse_win)
+    gamma = q_draft.shape[0]
+    dos, dls = [], []
+    for j in range(gamma):
+        o, l = draft_attn(q_draft[j], k_cache, v_cache, idx, count, t_ctx, j)
+        dos.append(o)
+        dls.append(l)
+    vo, vl = verify_attn(q_verify, k_cache, v_cache, t_ctx)
+    return dict(idx=idx, count=count, score=score, draft_o=np.stack(dos),
+                draft_lse=np.stack(dls), verify_o=vo, verify_lse=vl)
+
+
+def widen_bf16_bits(bits: np.ndarray) -> np.ndarray:
+    """Exact float64 value of bf16 bit patterns (uint16)."""
+    bits = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16
+    return bits.view(np.float32).astype(np.float64)

@@ -1,0 +1,83 @@
+"""Writes the hand-derived fixtures in this folder.
+
+Every expected value below is a closed form derived by hand (the derivation is
+stored in each fixture); nothing here calls the oracle or the CUDA path.
+Run:  python tests/golden/write_fixtures.py
+"""
+import json
+import math
+import os
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+FIXTURES = {
+    "attention_basis.json": {
+        "cite": "Sec. 3.1: p_S / p_L are softmax attention; closed form for basis keys",
+        "derivation": "d=4, scale=1/2. Keys e0,e1,e2; q = (2 ln 3) e0, so logits are (ln 3, 0, 0), "
+                      "probabilities (3/5, 1/5, 1/5), lse = ln 5. V rows (1,0,0,0), (0,1,0,0), (1,1,0,2) give "
+                      "o = 3/5 v0 + 1/5 v1 + 1/5 v2 = (0.8, 0.4, 0, 0.4).",
+        "q": [2 * math.log(3), 0, 0, 0],
+        "keys": [[1, 0, 0, 0], [0, 1, 0, 0], [0, 0, 1, 0]],
+        "values": [[1, 0, 0, 0], [0, 1, 0, 0], [1, 1, 0, 2]],
+        "scale": 0.5,
+        "o": [0.8, 0.4, 0.0, 0.4],
+        "lse": math.log(5),
+    },
+    "verify_causal.json": {
+        "cite": "Algorithm 2, Verify: the block's queries see the full cache with a causal mask inside the block",
+        "derivation": "t_ctx=2, n_q=2, one head, d=2 (scale 1/sqrt 2). Keys k0=k1=k3=(0,0), k2=(sqrt2 ln2, 0); "
+                      "q=(1,0) for both block queries. Query 0 (position 2) sees keys 0..2 with logits (0,0,ln2): "
+                      "p=(1/4,1/4,1/2), lse=ln4. Query 1 (position 3) sees keys 0..3 with logits (0,0,ln2,0): "
+                      "p=(1/5,1/5,2/5,1/5), lse=ln5. V rows (1,0),(0,1),(2,2),(4,0): o0=(1.25,1.25), o1=(1.8,1.0).",
+        "t_ctx": 2,
+        "q": [[1, 0], [1, 0]],
+        "keys": [[0, 0], [0, 0], [math.sqrt(2) * math.log(2), 0], [0, 0]],
+        "values": [[1, 0], [0, 1], [2, 2], [4, 0]],
+        "o": [[1.25, 1.25], [1.8, 1.0]],
+        "lse": [math.log(4), math.log(5)],
+    },
+    "window_scores_uniform.json": {
+        "cite": "Sec. 3.4: chunks scored by cumulative attention weight (window reading: causal rows over the "
+                "last W positions)",
+        "derivation": "t_ctx=3, W=2 (window rows at positions 1 and 2), one head, d=2, all keys zero. Row at "
+                      "position 1 spreads 1/2 over keys 0,1; row at position 2 spreads 1/3 over keys 0,1,2. "
+                      "lse=(ln2, ln3); score=(1/2+1/3, 1/2+1/3, 1/3).",
+        "t_ctx": 3,
+        "q_win": [[0.5, -1.0], [2.0, 0.25]],
+        "keys": [[0, 0], [0, 0], [0, 0]],
+        "lse": [math.log(2), math.log(3)],
+        "score": [5 / 6, 5 / 6, 1 / 3],
+    },
+    "selection_example.json": {
+        "cite": "Sec. 3.4 TopKChunks (top floor(B/s) by cumulative attention weight); token level with "
+                "sink/recent as in the graded workloads",
+        "derivation": "t_ctx=12, sink 2, recent 3, budget 8: middle = positions 2..8, 3 free slots. Middle scores "
+                      "(.5,.7,.2,.7,.9,.1,.7) at positions 2..8. Best is position 6 (.9); positions 3, 5, 8 tie at "
+                      ".7 and the lower two (3, 5) win. Keep = {0,1} + {3,5,6} + {9,10,11}. Chunk size 2: chunks "
+                      "[2,4)=1.2, [4,6)=.9, [6,8)=1.0, [8,9)=.7; one chunk fits (3//2) -> [2,4): keep "
+                      "{0,1,2,3,9,10,11}. Budget 12 >= t_ctx keeps all.",
+        "t_ctx": 12, "n_sink": 2, "n_recent": 3,
+        "score": [9, 9, 0.5, 0.7, 0.2, 0.7, 0.9, 0.1, 0.7, 5, 5, 5],
+        "cases": [
+            {"budget": 8, "chunk": 1, "keep": [0, 1, 3, 5, 6, 9, 10, 11]},
+            {"budget": 8, "chunk": 2, "keep": [0, 1, 2, 3, 9, 10, 11]},
+            {"budget": 12, "chunk": 1, "keep": list(range(12))},
+        ],
+    },
+    "combine_two_halves.json": {
+        "cite": "log-sum-exp merge of attention over disjoint key sets (split-K partials)",
+        "derivation": "Part A: keys with logits (0, 0) -> lse_A = ln2, o_A = mean of (1,0),(0,1) = (.5,.5). "
+                      "Part B: one key with logit ln2 -> lse_B = ln2, o_B = (3,1). Union: logits (0,0,ln2) -> "
+                      "p=(1/4,1/4,1/2), o = (1/4 + 3/2, 1/4 + 1/2) = (1.75, .75), lse = ln4.",
+        "o_part": [[[0.5, 0.5]], [[3.0, 1.0]]],
+        "lse_part": [[math.log(2)], [math.log(2)]],
+        "o": [[1.75, 0.75]],
+        "lse": [math.log(4)],
+    },
+}
+
+if __name__ == "__main__":
+    for name, obj in FIXTURES.items():
+        with open(os.path.join(HERE, name), "w") as f:
+            json.dump(obj, f, indent=1)
+    print(f"wrote {len(FIXTURES)} fixtures")
