@@ -1,0 +1,170 @@
+/*
+ * budgetdraft.h - C ABI of the speculative-step attention library (libbudgetdraft.so).
+ *
+ * One speculative step of BudgetDraft (arXiv 2606.00144, Algorithm 2) spends its
+ * KV-cache attention in three places, each an entry point below:
+ *   bd_select_budget  builds the drafter's sparse view K_S^sp(B) under a KV budget B
+ *                     (Sec. 3.4 TopKChunks; Algorithm 2, sparsify);
+ *   bd_draft_attn     one of the gamma drafter decode passes over that view
+ *                     (Algorithm 2, Draft);
+ *   bd_verify_attn    the verifier's (gamma+1)-query pass over the full cache with a
+ *                     causal mask inside the draft block (Algorithm 2, Verify);
+ *   bd_combine        the log-sum-exp merge of attention computed over disjoint key
+ *                     sets (split-K partials).
+ *
+ * Conventions shared by every call
+ *   - All tensor arguments are DEVICE pointers owned by the caller; the library
+ *     never allocates, frees or keeps a pointer after a call returns.
+ *   - bf16 tensors are IEEE bfloat16 (raw 16-bit), fp32 are IEEE float, int32 are
+ *     int32_t.  Every tensor is dense row-major in the order written, and every
+ *     pointer must be 16-byte aligned.
+ *   - KV caches are bf16 [batch, h_kv, t_cap, head_dim].  Rows hold post-RoPE keys
+ *     and values: position p of (sequence b, KV head g) is row p.  Positions
+ *     [0, t_ctx) are the context; rows t_ctx, t_ctx+1, ... hold the tokens of the
+ *     current draft / verify block.
+ *   - GQA: query head h reads KV head h / (h_q / h_kv).
+ *   - Softmax scale is 1/sqrt(head_dim); every lse is a natural logarithm.
+ *   - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream).  A call returns BD_OK or a negative bd_status after validating every
+ *     argument on the host BEFORE any launch; a failed launch returns BD_ERR_CUDA.
+ *   - Workspace: `ws` is a caller-owned device buffer of at least
+ *     bd_workspace_size(...) bytes for that call.  It must be zero-filled once
+ *     before its first use; calls that finish leave its counter words zero again,
+ *     so it can be reused without clearing.  Calls that share one workspace must
+ *     be ordered (same stream, or synchronised).  Kernels record device-side
+ *     errors (a bounded wait that ran out) in the workspace's status word, which
+ *     bd_workspace_status() reads.
+ *   - Supported: head_dim 64 or 128; h_q % h_kv == 0.
+ */
+#ifndef BUDGETDRAFT_H
+#define BUDGETDRAFT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum bd_status {
+  BD_OK = 0,
+  BD_ERR_INVALID_ARG = -1,  /* a null pointer, a size out of range, inconsistent shape  */
+  BD_ERR_UNSUPPORTED = -2,  /* valid but not implemented (head_dim, too many queries)    */
+  BD_ERR_MISALIGNED = -3,   /* a tensor pointer is not 16-byte aligned                   */
+  BD_ERR_WORKSPACE = -4,    /* ws is NULL or smaller than bd_workspace_size()            */
+  BD_ERR_CUDA = -5,         /* a CUDA runtime call or a launch failed                    */
+  BD_ERR_TIMEOUT = -6       /* device side: a bounded wait ran out (status word only)    */
+} bd_status;
+
+/* Problem shape of one layer's cache.  The caches are [batch, h_kv, t_cap, head_dim]. */
+typedef struct bd_shape {
+  int32_t batch;     /* sequences                                   */
+  int32_t h_q;       /* query heads                                 */
+  int32_t h_kv;      /* KV heads, divides h_q                        */
+  int32_t head_dim;  /* d: 64 or 128                                 */
+  int32_t t_ctx;     /* context length T (cached prefix positions)   */
+  int32_t t_cap;     /* rows per (sequence, KV head) in the arrays   */
+} bd_shape;
+
+/* Operation codes for bd_workspace_size. */
+enum { BD_OP_SELECT = 1, BD_OP_DRAFT = 2, BD_OP_VERIFY = 3 };
+
+/*
+ * Workspace bytes needed by one operation on `shape` (0 on invalid input).
+ *   BD_OP_SELECT: budget = B, n_q = window W (window queries per head);
+ *   BD_OP_DRAFT:  budget = B, n_q = the largest step_j + 1 that will be passed;
+ *   BD_OP_VERIFY: budget ignored, n_q = queries per head in the block.
+ * The size depends on the current device's SM count.  Sizes for different ops may
+ * be satisfied by one buffer of the largest of them.
+ */
+size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q);
+
+/*
+ * KV-budget selection: the sparse drafter view K_S^sp(B) of every (sequence, KV
+ * head).  Sec. 3.4 of the paper keeps the top floor(B/s) chunks of the prefix by
+ * cumulative attention weight; this library reads "cumulative attention weight" of
+ * position k as
+ *     score[k] = sum over the group's query heads h and window rows w with k <= p_w
+ *                of exp(q_{h,w} . k_k / sqrt(d) - lse_{h,w}),
+ * the summed causal softmax probability that the last W context queries (window
+ * row w sits at position p_w = t_ctx - W + w) put on key k.
+ *   keep = [0, n_sink)  U  [t_ctx - n_recent, t_ctx)
+ *          U  best of the middle [n_sink, t_ctx - n_recent):
+ *               chunk == 1: the top (budget - n_sink - n_recent) positions by score;
+ *               chunk == s > 1: the top floor((budget - n_sink - n_recent)/s) chunks,
+ *                 chunk c = positions [c s, c s + s) within the middle, scored by the
+ *                 sum of its members;
+ *          ties go to the lower position (chunk).  If budget >= t_ctx, keep = [0, t_ctx).
+ *
+ *   k_cache     bf16 [batch, h_kv, t_cap, d]; rows [0, t_ctx) are read.
+ *   q_window    bf16 [batch, h_q, window, d]: queries of positions t_ctx-W .. t_ctx-1.
+ *   window_lse  fp32 [batch, h_q, window]: each window row's softmax normaliser over
+ *               keys [0, p_w] (carried from the step that verified that token), or
+ *               NULL to have it computed here (reads K a second time).
+ *   idx_out     int32 [batch, h_kv, budget]: kept positions ascending, then -1 padding.
+ *   count_out   int32 [batch, h_kv]: number of kept positions.
+ * Constraints: 1 <= window <= t_ctx, (h_q/h_kv)*window <= 256, n_sink, n_recent >= 0,
+ * n_sink + n_recent <= budget when budget < t_ctx, chunk >= 1, t_cap >= t_ctx.
+ */
+int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_window,
+                     const float* window_lse, int window, int budget, int n_sink, int n_recent,
+                     int chunk, int32_t* idx_out, int32_t* count_out, void* ws, size_t ws_bytes,
+                     void* stream);
+
+/*
+ * Drafter decode pass j (0-based) over the sparse view (Algorithm 2, Draft):
+ * each query head h of sequence b attends to rows idx[b, g, 0:count[b, g]] and to
+ * the drafted rows t_ctx .. t_ctx + step_j of its KV head g (the drafter's own
+ * tokens are appended to its sparse cache, Algorithm 2, Update).
+ *   q        bf16 [batch, h_q, d]
+ *   idx      int32 [batch, h_kv, budget] positions in [0, t_ctx) (as written by
+ *            bd_select_budget; entries past count are ignored); count int32 [batch, h_kv]
+ *            with 0 <= count <= budget.
+ *   o_out    bf16 [batch, h_q, d];  lse_out fp32 [batch, h_q] (may be NULL).
+ * Constraints: step_j >= 0, t_ctx + step_j < t_cap.
+ */
+int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
+                  const int32_t* idx, const int32_t* count, int budget, int step_j, void* o_out,
+                  float* lse_out, void* ws, size_t ws_bytes, void* stream);
+
+/*
+ * Verifier block attention (Algorithm 2, Verify): query i (0 <= i < n_q) of head h
+ * sits at position t_ctx + i and attends to keys [0, t_ctx + i] of its KV head.
+ *   q        bf16 [batch, h_q, n_q, d]
+ *   o_out    bf16 [batch, h_q, n_q, d], or NULL to compute lse only (V not read);
+ *   lse_out  fp32 [batch, h_q, n_q] (may be NULL when o_out is not).
+ * Constraints: 1 <= n_q, t_ctx + n_q <= t_cap, (h_q/h_kv)*n_q <= 96 (<= 128 when
+ * o_out is NULL).
+ */
+int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_cache,
+                   const void* v_cache, void* o_out, float* lse_out, void* ws, size_t ws_bytes,
+                   void* stream);
+
+/*
+ * Log-sum-exp merge of attention over disjoint key sets: with L = log sum_s exp(lse_s),
+ *   o = sum_s exp(lse_s - L) o_s,   lse = L.
+ * A part with lse = -inf is empty and contributes nothing; rows whose parts are all
+ * empty give o = 0 and lse = -inf.
+ *   o_part   fp32 [n_split, rows, d], each row normalised over its own key set;
+ *   lse_part fp32 [n_split, rows];
+ *   o_out    bf16 [rows, d];  lse_out fp32 [rows] (may be NULL).
+ * Constraints: n_split >= 1, rows >= 0 (0 is a no-op), head_dim 64 or 128.
+ */
+int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows, int head_dim,
+               void* o_out, float* lse_out, void* stream);
+
+/*
+ * Reads (and clears) the device status word of a workspace: BD_OK, or the first
+ * device-side error recorded by a kernel since the last read.  Synchronises
+ * `stream`.  Returns BD_ERR_INVALID_ARG for a NULL ws, BD_ERR_CUDA if the copy fails.
+ */
+int bd_workspace_status(void* ws, void* stream);
+
+/* Static description of a status code. */
+const char* bd_strerror(int status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BUDGETDRAFT_H */

@@ -120,10 +120,16 @@ def verify_attn(q: np.ndarray, k_cache: np.ndarray, v_cache: np.ndarray, t_ctx: 
     for bi in range(b):
         for h in range(h_q):
             kv = h // group
+            keys = k_cache[bi, kv, : t_ctx + n_q]
+            vals = v_cache[bi, kv, : t_ctx + n_q]
+            logits = scale * (q[bi, h] @ keys.T)          # [n_q, t_ctx + n_q]
             for i in range(n_q):
-                last = t_ctx + i
-                o[bi, h, i], lse[bi, h, i] = attention(
-                    q[bi, h, i], k_cache[bi, kv, : last + 1], v_cache[bi, kv, : last + 1], scale)
+                s = logits[i, : t_ctx + i + 1]             # causal: keys [0, t_ctx + i]
+                m = s.max()
+                e = np.exp(s - m)
+                l = e.sum()
+                o[bi, h, i] = (e @ vals[: t_ctx + i + 1]) / l
+                lse[bi, h, i] = m + math.log(l)
     return o, lse
 
 
@@ -179,8 +185,9 @@ def window_lse(q_win: np.ndarray, k_cache: np.ndarray, t_ctx: int):
     for bi in range(b):
         for h in range(h_q):
             kv = h // group
+            logits = scale * (q_win[bi, h] @ k_cache[bi, kv, :t_ctx].T)     # [W, t_ctx]
             for w in range(window):
-                s = scale * (k_cache[bi, kv, : pos[w] + 1] @ q_win[bi, h, w])
+                s = logits[w, : pos[w] + 1]
                 m = s.max()
                 lse[bi, h, w] = m + math.log(np.exp(s - m).sum())
     return lse
@@ -198,16 +205,16 @@ def window_scores(q_win: np.ndarray, k_cache: np.ndarray, lse_win: np.ndarray, t
     group = h_q // h_kv
     scale = 1.0 / math.sqrt(d)
     pos = window_positions(t_ctx, window)
+    causal = np.arange(t_ctx)[None, :] <= pos[:, None]                  # [W, t_ctx]
     score = np.zeros((b, h_kv, t_ctx), dtype=np.float64)
     for bi in range(b):
         for kv in range(h_kv):
             keys = k_cache[bi, kv, :t_ctx]
             for g in range(group):
                 h = kv * group + g
-                for w in range(window):
-                    p = np.exp(scale * (keys @ q_win[bi, h, w]) - lse_win[bi, h, w])
-                    p[pos[w] + 1:] = 0.0          # causal: row w sees [0, p_w]
-                    score[bi, kv] += p
+                p = np.exp(scale * (q_win[bi, h] @ keys.T) - lse_win[bi, h][:, None])   # [W, t_ctx]
+                p[~causal] = 0.0                                  # row w sees [0, p_w]
+                score[bi, kv] += p.sum(axis=0)
     return score
 
 

@@ -1,0 +1,28 @@
+"""GB300 (sm_103a) speculative-step attention of BudgetDraft (arXiv 2606.00144).
+
+The hot path (KV-budget selection, gamma drafter decode passes over the sparse view, the
+verifier's causal block pass and the log-sum-exp merge) lives in libbudgetdraft.so
+(hand-written CUDA, C ABI in include/budgetdraft.h).  This package holds its build step,
+a thin ctypes binding, a step runner and the seeded synthetic workloads.
+"""
+
+from .binding import (  # noqa: F401
+    BD_OP_DRAFT,
+    BD_OP_SELECT,
+    BD_OP_VERIFY,
+    BdShape,
+    BudgetDraftError,
+    Workspace,
+    bd_combine,
+    bd_draft_attn,
+    bd_select_budget,
+    bd_strerror,
+    bd_verify_attn,
+    bd_workspace_size,
+    bd_workspace_status,
+    library,
+    make_shape,
+    shape_of,
+)
+from .build import LIB_PATH, build  # noqa: F401
+from .step import SpecStep  # noqa: F401

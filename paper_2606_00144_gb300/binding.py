@@ -1,0 +1,162 @@
+"""Thin ctypes binding of libbudgetdraft (include/budgetdraft.h).
+
+Argument marshalling only: every computation runs in the library's CUDA kernels.  torch
+tensors provide device memory and the current CUDA stream.  There is no fallback: if
+the library is not built, or an argument is rejected, these functions raise.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from .build import LIB_PATH
+
+BD_OK = 0
+BD_OP_SELECT, BD_OP_DRAFT, BD_OP_VERIFY = 1, 2, 3
+
+
+class BdShape(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int32), ("h_q", ctypes.c_int32), ("h_kv", ctypes.c_int32),
+                ("head_dim", ctypes.c_int32), ("t_ctx", ctypes.c_int32), ("t_cap", ctypes.c_int32)]
+
+    def __repr__(self):
+        return (f"BdShape(batch={self.batch}, h_q={self.h_q}, h_kv={self.h_kv}, head_dim={self.head_dim}, "
+                f"t_ctx={self.t_ctx}, t_cap={self.t_cap})")
+
+
+class BudgetDraftError(RuntimeError):
+    def __init__(self, func, status):
+        self.status = status
+        super().__init__(f"{func} failed: {bd_strerror(status)} ({status})")
+
+
+_lib = None
+_P = ctypes.c_void_p
+_SHAPE = ctypes.POINTER(BdShape)
+_SIGNATURES = {
+    "bd_workspace_size": (ctypes.c_size_t, [_SHAPE, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
+    "bd_select_budget": (ctypes.c_int, [_SHAPE, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                        ctypes.c_int, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
+    "bd_draft_attn": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P,
+                                     ctypes.c_size_t, _P]),
+    "bd_verify_attn": (ctypes.c_int, [_SHAPE, _P, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
+    "bd_combine": (ctypes.c_int, [_P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P, _P]),
+    "bd_workspace_status": (ctypes.c_int, [_P, _P]),
+    "bd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+}
+
+
+def library():
+    """Load libbudgetdraft.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(f"{LIB_PATH} is not built; run paper_2606_00144_gb300.build.build() first")
+        lib = ctypes.CDLL(LIB_PATH)
+        for name, (res, args) in _SIGNATURES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+def exported_symbols():
+    return list(_SIGNATURES)
+
+
+def bd_strerror(status: int) -> str:
+    return library().bd_strerror(int(status)).decode()
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(name, status):
+    if status != BD_OK:
+        raise BudgetDraftError(name, status)
+
+
+def make_shape(batch, h_q, h_kv, head_dim, t_ctx, t_cap) -> BdShape:
+    return BdShape(int(batch), int(h_q), int(h_kv), int(head_dim), int(t_ctx), int(t_cap))
+
+
+def shape_of(k_cache: torch.Tensor, h_q: int, t_ctx: int) -> BdShape:
+    b, h_kv, t_cap, d = k_cache.shape
+    return make_shape(b, h_q, h_kv, d, t_ctx, t_cap)
+
+
+def bd_workspace_size(shape: BdShape, op: int, budget: int, n_q: int) -> int:
+    return int(library().bd_workspace_size(ctypes.byref(shape), op, int(budget), int(n_q)))
+
+
+class Workspace:
+    """A zero-filled device buffer sized for a set of operations (see bd_workspace_size)."""
+
+    def __init__(self, nbytes: int, device=None):
+        self.nbytes = int(max(nbytes, 512))
+        self.buf = torch.zeros(self.nbytes, dtype=torch.uint8, device=device or "cuda")
+
+    @classmethod
+    def for_step(cls, shape: BdShape, budget: int, window: int, gamma: int, device=None):
+        sizes = [bd_workspace_size(shape, BD_OP_SELECT, budget, window),
+                 bd_workspace_size(shape, BD_OP_DRAFT, budget, gamma),
+                 bd_workspace_size(shape, BD_OP_VERIFY, budget, gamma + 1)]
+        if min(sizes) == 0:
+            raise BudgetDraftError("bd_workspace_size", -1)
+        return cls(max(sizes), device)
+
+    @property
+    def ptr(self):
+        return self.buf.data_ptr()
+
+    def status(self, stream=None) -> int:
+        return int(library().bd_workspace_status(self.ptr, _stream(stream)))
+
+
+def bd_select_budget(shape, k_cache, q_window, window_lse, window, budget, n_sink, n_recent, chunk,
+                     idx_out, count_out, ws: Workspace, stream=None):
+    st = library().bd_select_budget(ctypes.byref(shape), _ptr(k_cache), _ptr(q_window), _ptr(window_lse),
+                                    int(window), int(budget), int(n_sink), int(n_recent), int(chunk),
+                                    _ptr(idx_out), _ptr(count_out), ws.ptr, ws.nbytes, _stream(stream))
+    _check("bd_select_budget", st)
+
+
+def bd_draft_attn(shape, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
+                  ws: Workspace, stream=None):
+    st = library().bd_draft_attn(ctypes.byref(shape), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(idx),
+                                 _ptr(count), int(budget), int(step_j), _ptr(o_out), _ptr(lse_out), ws.ptr,
+                                 ws.nbytes, _stream(stream))
+    _check("bd_draft_attn", st)
+
+
+def bd_verify_attn(shape, q, n_q, k_cache, v_cache, o_out, lse_out, ws: Workspace, stream=None):
+    st = library().bd_verify_attn(ctypes.byref(shape), _ptr(q), int(n_q), _ptr(k_cache), _ptr(v_cache),
+                                  _ptr(o_out), _ptr(lse_out), ws.ptr, ws.nbytes, _stream(stream))
+    _check("bd_verify_attn", st)
+
+
+def bd_combine(o_part, lse_part, n_split, rows, head_dim, o_out, lse_out, stream=None):
+    st = library().bd_combine(_ptr(o_part), _ptr(lse_part), int(n_split), int(rows), int(head_dim),
+                              _ptr(o_out), _ptr(lse_out), _stream(stream))
+    _check("bd_combine", st)
+
+
+def bd_workspace_status(ws: Workspace, stream=None) -> int:
+    return ws.status(stream)

@@ -1,0 +1,244 @@
+// The C ABI of libbudgetdraft (include/budgetdraft.h): argument validation on the host
+// before any launch, workspace layout, and dispatch to the kernels.
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <mutex>
+
+#include "bd_common.cuh"
+#include "bd_internal.h"
+
+namespace bd {
+
+int current_sm_count() {
+  static int cache[256] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+  if (dev < 256 && cache[dev] > 0) return cache[dev];
+  int n = 0;
+  if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+  if (dev < 256) cache[dev] = n;
+  return n;
+}
+
+size_t ws_counters_offset() { return kWsHeaderBytes; }
+size_t ws_region_offset(int units) { return kWsHeaderBytes + align_up((size_t)units * 4, 256); }
+
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+cudaError_t make_cache_map(CUtensorMap* map, const void* base, int units, int t_cap, int n_rows, int head_dim,
+                           int box_rows) {
+  auto fn = encode_fn();
+  if (!fn) return cudaErrorNotSupported;
+  const cuuint64_t dims[3] = {(cuuint64_t)head_dim, (cuuint64_t)n_rows, (cuuint64_t)units};
+  const cuuint64_t strides[2] = {(cuuint64_t)head_dim * 2, (cuuint64_t)t_cap * head_dim * 2};
+  const cuuint32_t box[3] = {64, (cuuint32_t)box_rows, 1};
+  const cuuint32_t estride[3] = {1, 1, 1};
+  const CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+                        estride, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                        CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  return r == CUDA_SUCCESS ? cudaSuccess : cudaErrorInvalidValue;
+}
+
+}  // namespace bd
+
+using namespace bd;
+
+namespace {
+
+bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+int check_shape(const bd_shape* s) {
+  if (!s) return BD_ERR_INVALID_ARG;
+  if (s->batch < 1 || s->h_q < 1 || s->h_kv < 1 || s->h_q % s->h_kv != 0 || s->t_ctx < 1 || s->t_cap < s->t_ctx)
+    return BD_ERR_INVALID_ARG;
+  if (s->head_dim != 64 && s->head_dim != 128) return BD_ERR_UNSUPPORTED;
+  // every per-unit row offset must stay addressable by the TMA (rows < 2^31)
+  if ((long long)s->batch * s->h_kv * s->t_cap >= (1LL << 31)) return BD_ERR_UNSUPPORTED;
+  return BD_OK;
+}
+
+int check_tensor(const void* p, uintptr_t align) {
+  if (!p) return BD_ERR_INVALID_ARG;
+  return aligned(p, align) ? BD_OK : BD_ERR_MISALIGNED;
+}
+
+int map_cuda(cudaError_t e) { return e == cudaSuccess ? BD_OK : BD_ERR_CUDA; }
+
+int* status_word(void* ws) { return static_cast<int*>(ws); }
+int* counters(void* ws) { return reinterpret_cast<int*>(static_cast<uint8_t*>(ws) + ws_counters_offset()); }
+void* region(void* ws, int units) { return static_cast<uint8_t*>(ws) + ws_region_offset(units); }
+
+bool group_supported_by_draft(int g) { return g == 1 || g == 2 || g == 4 || g == 8; }
+
+size_t verify_ws(const bd_shape& s, int n_q, bool with_v, bool* ok) {
+  VerifyPlan vp;
+  *ok = verify_plan(s, n_q, with_v, &vp);
+  return *ok ? ws_region_offset(s.batch * s.h_kv) + verify_partials_bytes(s, vp) : 0;
+}
+
+}  // namespace
+
+#define BD_TRY(x)                  \
+  do {                             \
+    const int _st = (x);           \
+    if (_st != BD_OK) return _st;  \
+  } while (0)
+
+extern "C" {
+
+size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q) {
+  if (check_shape(shape) != BD_OK) return 0;
+  const bd_shape& s = *shape;
+  const int units = s.batch * s.h_kv;
+  switch (op) {
+    case BD_OP_SELECT: {
+      if (n_q < 1 || n_q > s.t_ctx || budget < 1) return 0;
+      SelectPlan sp;
+      if (!select_plan(s, n_q, budget, 0, 0, 1, &sp)) return 0;
+      return ws_region_offset(units) + select_region_bytes(s, sp);
+    }
+    case BD_OP_DRAFT: {
+      if (n_q < 1 || budget < 1) return 0;
+      DraftPlan dp;
+      if (!draft_plan(s, budget, n_q, &dp)) return 0;
+      return ws_region_offset(units) + draft_partials_bytes(s, dp);
+    }
+    case BD_OP_VERIFY: {
+      if (n_q < 1) return 0;
+      bool ok_v = false, ok_l = false;
+      const size_t a = verify_ws(s, n_q, true, &ok_v);
+      const size_t b = verify_ws(s, n_q, false, &ok_l);
+      if (!ok_v && !ok_l) return 0;
+      return std::max(a, b);
+    }
+    default:
+      return 0;
+  }
+}
+
+int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_window, const float* window_lse,
+                     int window, int budget, int n_sink, int n_recent, int chunk, int32_t* idx_out,
+                     int32_t* count_out, void* ws, size_t ws_bytes, void* stream) {
+  BD_TRY(check_shape(shape));
+  const bd_shape& s = *shape;
+  BD_TRY(check_tensor(k_cache, 16));
+  BD_TRY(check_tensor(q_window, 16));
+  if (window_lse) BD_TRY(check_tensor(window_lse, 4));
+  BD_TRY(check_tensor(idx_out, 4));
+  BD_TRY(check_tensor(count_out, 4));
+  if (window < 1 || window > s.t_ctx || budget < 1 || n_sink < 0 || n_recent < 0 || chunk < 1)
+    return BD_ERR_INVALID_ARG;
+  if (budget < s.t_ctx && n_sink + n_recent > budget) return BD_ERR_INVALID_ARG;
+  if ((s.h_q / s.h_kv) * window > 256) return BD_ERR_UNSUPPORTED;
+  SelectPlan sp;
+  if (!select_plan(s, window, budget, n_sink, n_recent, chunk, &sp)) return BD_ERR_UNSUPPORTED;
+  if (!ws) return BD_ERR_WORKSPACE;
+  if (!aligned(ws, 256)) return BD_ERR_MISALIGNED;
+  const int units = s.batch * s.h_kv;
+  if (ws_bytes < ws_region_offset(units) + select_region_bytes(s, sp)) return BD_ERR_WORKSPACE;
+  return map_cuda(launch_select(s, sp, k_cache, q_window, window_lse, window, budget, n_sink, n_recent, chunk,
+                                idx_out, count_out, region(ws, units), counters(ws), status_word(ws),
+                                static_cast<cudaStream_t>(stream)));
+}
+
+int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
+                  const int32_t* idx, const int32_t* count, int budget, int step_j, void* o_out, float* lse_out,
+                  void* ws, size_t ws_bytes, void* stream) {
+  BD_TRY(check_shape(shape));
+  const bd_shape& s = *shape;
+  BD_TRY(check_tensor(q, 16));
+  BD_TRY(check_tensor(k_cache, 16));
+  BD_TRY(check_tensor(v_cache, 16));
+  BD_TRY(check_tensor(idx, 4));
+  BD_TRY(check_tensor(count, 4));
+  BD_TRY(check_tensor(o_out, 16));
+  if (lse_out) BD_TRY(check_tensor(lse_out, 4));
+  if (budget < 1 || step_j < 0 || (long long)s.t_ctx + step_j >= s.t_cap) return BD_ERR_INVALID_ARG;
+  if (!group_supported_by_draft(s.h_q / s.h_kv)) return BD_ERR_UNSUPPORTED;
+  DraftPlan dp;
+  if (!draft_plan(s, budget, step_j + 1, &dp)) return BD_ERR_UNSUPPORTED;
+  if (!ws) return BD_ERR_WORKSPACE;
+  if (!aligned(ws, 256)) return BD_ERR_MISALIGNED;
+  const int units = s.batch * s.h_kv;
+  if (ws_bytes < ws_region_offset(units) + draft_partials_bytes(s, dp)) return BD_ERR_WORKSPACE;
+  return map_cuda(launch_draft(s, dp, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
+                               region(ws, units), counters(ws), status_word(ws), static_cast<cudaStream_t>(stream)));
+}
+
+int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_cache, const void* v_cache,
+                   void* o_out, float* lse_out, void* ws, size_t ws_bytes, void* stream) {
+  BD_TRY(check_shape(shape));
+  const bd_shape& s = *shape;
+  BD_TRY(check_tensor(q, 16));
+  BD_TRY(check_tensor(k_cache, 16));
+  if (o_out) {
+    BD_TRY(check_tensor(v_cache, 16));
+    BD_TRY(check_tensor(o_out, 16));
+  }
+  if (lse_out) BD_TRY(check_tensor(lse_out, 4));
+  if (!o_out && !lse_out) return BD_ERR_INVALID_ARG;
+  if (n_q < 1 || (long long)s.t_ctx + n_q > s.t_cap) return BD_ERR_INVALID_ARG;
+  const bool with_v = o_out != nullptr;
+  const int nq_rows = (s.h_q / s.h_kv) * n_q;
+  if (nq_rows > (with_v ? 96 : 128)) return BD_ERR_UNSUPPORTED;
+  VerifyPlan vp;
+  if (!verify_plan(s, n_q, with_v, &vp)) return BD_ERR_UNSUPPORTED;
+  if (!ws) return BD_ERR_WORKSPACE;
+  if (!aligned(ws, 256)) return BD_ERR_MISALIGNED;
+  const int units = s.batch * s.h_kv;
+  if (ws_bytes < ws_region_offset(units) + verify_partials_bytes(s, vp)) return BD_ERR_WORKSPACE;
+  return map_cuda(launch_verify(s, vp, n_q, q, k_cache, v_cache, o_out, lse_out, region(ws, units), counters(ws),
+                                status_word(ws), static_cast<cudaStream_t>(stream)));
+}
+
+int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows, int head_dim, void* o_out,
+               float* lse_out, void* stream) {
+  if (n_split < 1 || rows < 0) return BD_ERR_INVALID_ARG;
+  if (head_dim != 64 && head_dim != 128) return BD_ERR_UNSUPPORTED;
+  if (rows == 0) return BD_OK;
+  BD_TRY(check_tensor(o_part, 16));
+  BD_TRY(check_tensor(lse_part, 4));
+  BD_TRY(check_tensor(o_out, 16));
+  if (lse_out) BD_TRY(check_tensor(lse_out, 4));
+  if ((long long)n_split * rows * head_dim >= (1LL << 40)) return BD_ERR_UNSUPPORTED;
+  return map_cuda(launch_combine(o_part, lse_part, n_split, rows, head_dim, o_out, lse_out,
+                                 static_cast<cudaStream_t>(stream)));
+}
+
+int bd_workspace_status(void* ws, void* stream) {
+  if (!ws) return BD_ERR_INVALID_ARG;
+  int host = 0;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(&host, ws, sizeof(int), cudaMemcpyDeviceToHost, st) != cudaSuccess) return BD_ERR_CUDA;
+  if (cudaMemsetAsync(ws, 0, sizeof(int), st) != cudaSuccess) return BD_ERR_CUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return BD_ERR_CUDA;
+  return host;
+}
+
+const char* bd_strerror(int status) {
+  switch (status) {
+    case BD_OK: return "ok";
+    case BD_ERR_INVALID_ARG: return "invalid argument";
+    case BD_ERR_UNSUPPORTED: return "unsupported shape or option";
+    case BD_ERR_MISALIGNED: return "misaligned pointer";
+    case BD_ERR_WORKSPACE: return "workspace missing or too small";
+    case BD_ERR_CUDA: return "CUDA runtime or launch error";
+    case BD_ERR_TIMEOUT: return "device-side bounded wait timed out";
+    default: return "unknown status";
+  }
+}
+
+}  // extern "C"

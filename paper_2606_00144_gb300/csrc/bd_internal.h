@@ -1,0 +1,87 @@
+// Host-side plumbing shared by the translation units of libbudgetdraft: launch plans,
+// workspace layout, tensor-map encoding and per-kernel launchers.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "budgetdraft.h"
+
+namespace bd {
+
+// ---------------------------------------------------------------------------- device facts
+int current_sm_count();   // SMs of the current device (cached per device)
+
+// ---------------------------------------------------------------------------- workspace
+// [0, 256): status word; [256, 256 + units*4 rounded to 256): per-unit arrival counters;
+// then the op-specific region.
+size_t ws_counters_offset();
+size_t ws_region_offset(int units);
+
+// ---------------------------------------------------------------------------- verify
+struct VerifyPlan {
+  int nq_rows;          // query rows per (sequence, KV head) = group * n_q
+  int nt, wq;           // n-tiles per warp, warp groups along queries
+  int n_tiles;          // 64-key tiles over [0, t_ctx + n_q)
+  int tiles_per_split;
+  int n_split;
+  int stages;
+  size_t smem_bytes;
+  bool with_v;
+};
+bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan);
+size_t verify_partials_bytes(const bd_shape& s, const VerifyPlan& plan);
+// q/o/lse as in bd_verify_attn; ws_region points at the op region, counters/status into ws.
+cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, const void* q,
+                          const void* k_cache, const void* v_cache, void* o_out, float* lse_out,
+                          void* ws_region, int* counters, int* status, cudaStream_t stream);
+
+// ---------------------------------------------------------------------------- draft
+struct DraftPlan {
+  int n_entries_max;    // budget + step_j + 1
+  int n_split;
+  int rows_per_split;
+};
+bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan);
+size_t draft_partials_bytes(const bd_shape& s, const DraftPlan& plan);
+cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q, const void* k_cache,
+                         const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
+                         int step_j, void* o_out, float* lse_out, void* ws_region, int* counters,
+                         int* status, cudaStream_t stream);
+
+// ---------------------------------------------------------------------------- select
+struct SelectPlan {
+  bool keep_all;        // budget >= t_ctx
+  bool need_scores;     // some middle position (chunk) must be ranked
+  int nq_rows, nq_pad;  // window query rows per KV head (padded to 16)
+  int n_mid, n_mid_pad;
+  int tiles_per_unit, total_tiles, grid, tiles_per_cta;
+  int stages;
+  uint32_t tmem_cols;
+  size_t smem_bytes;
+  size_t score_bytes, lse_bytes;
+  VerifyPlan lse_plan;  // self mode: window LSE through the verify kernel (lse only)
+};
+bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_recent, int chunk,
+                 SelectPlan* plan);
+size_t select_region_bytes(const bd_shape& s, const SelectPlan& plan);
+cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void* k_cache,
+                          const void* q_window, const float* window_lse, int window, int budget,
+                          int n_sink, int n_recent, int chunk, int32_t* idx_out, int32_t* count_out,
+                          void* ws_region, int* counters, int* status, cudaStream_t stream);
+
+// ---------------------------------------------------------------------------- combine
+cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_split, int rows,
+                           int head_dim, void* o_out, float* lse_out, cudaStream_t stream);
+int combine_rows_per_block(int n_split);
+
+// ---------------------------------------------------------------------------- TMA maps
+// 3-D map over a [units, rows_total (stride t_cap), head_dim] bf16 cache: only rows
+// [0, n_rows) of each unit are addressable (the rest reads as zero).  Box = 64 columns x
+// box_rows rows x 1 unit, 128-byte swizzle.
+cudaError_t make_cache_map(CUtensorMap* map, const void* base, int units, int t_cap, int n_rows,
+                           int head_dim, int box_rows);
+
+}  // namespace bd

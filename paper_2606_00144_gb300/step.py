@@ -1,0 +1,66 @@
+"""One speculative step's attention through the C ABI (Algorithm 2: sparsify, Draft x gamma,
+Verify), with preallocated outputs and workspace so the step can be captured in a CUDA graph."""
+
+from __future__ import annotations
+
+import torch
+
+from . import binding as B
+
+
+class SpecStep:
+    """Runs bd_select_budget, gamma x bd_draft_attn and bd_verify_attn for one layer.
+
+    The same object may serve many layers of one shape (the workspace is reused; calls
+    on one stream are ordered)."""
+
+    def __init__(self, batch, h_q, h_kv, head_dim, t_ctx, t_cap, budget, n_sink, n_recent,
+                 window=32, gamma=5, chunk=1, device="cuda"):
+        self.shape = B.make_shape(batch, h_q, h_kv, head_dim, t_ctx, t_cap)
+        self.budget, self.n_sink, self.n_recent = budget, n_sink, n_recent
+        self.window, self.gamma, self.chunk = window, gamma, chunk
+        self.ws = B.Workspace.for_step(self.shape, budget, window, gamma, device)
+        dev = torch.device(device)
+        self.idx = torch.empty(batch, h_kv, budget, dtype=torch.int32, device=dev)
+        self.count = torch.empty(batch, h_kv, dtype=torch.int32, device=dev)
+        self.draft_o = torch.empty(gamma, batch, h_q, head_dim, dtype=torch.bfloat16, device=dev)
+        self.draft_lse = torch.empty(gamma, batch, h_q, dtype=torch.float32, device=dev)
+        self.verify_o = torch.empty(batch, h_q, gamma + 1, head_dim, dtype=torch.bfloat16, device=dev)
+        self.verify_lse = torch.empty(batch, h_q, gamma + 1, dtype=torch.float32, device=dev)
+
+    @classmethod
+    def for_workload(cls, wl, budget=None, n_recent=None, chunk=1, device="cuda"):
+        b = wl.budget if budget is None else budget
+        r = wl.n_recent if n_recent is None else n_recent
+        return cls(wl.batch, wl.h_q, wl.h_kv, wl.head_dim, wl.t_ctx, wl.t_cap, b, wl.n_sink, r,
+                   wl.window, wl.gamma, chunk, device)
+
+    def select(self, k_cache, q_win, window_lse=None, stream=None):
+        B.bd_select_budget(self.shape, k_cache, q_win, window_lse, self.window, self.budget, self.n_sink,
+                           self.n_recent, self.chunk, self.idx, self.count, self.ws, stream)
+
+    def draft(self, j, q_j, k_cache, v_cache, stream=None):
+        B.bd_draft_attn(self.shape, q_j, k_cache, v_cache, self.idx, self.count, self.budget, j,
+                        self.draft_o[j], self.draft_lse[j], self.ws, stream)
+
+    def verify(self, q_verify, k_cache, v_cache, stream=None):
+        B.bd_verify_attn(self.shape, q_verify, self.gamma + 1, k_cache, v_cache, self.verify_o,
+                         self.verify_lse, self.ws, stream)
+
+    def run(self, k_cache, v_cache, q_win, q_draft, q_verify, window_lse=None, stream=None):
+        self.select(k_cache, q_win, window_lse, stream)
+        for j in range(self.gamma):
+            self.draft(j, q_draft[j], k_cache, v_cache, stream)
+        self.verify(q_verify, k_cache, v_cache, stream)
+
+    def window_lse(self, k_cache, q_win, out=None, stream=None):
+        """LSE of the window queries over their causal prefixes, computed by the verify
+        kernel (what a previous verify / prefill step leaves behind for carry mode)."""
+        sh = B.make_shape(self.shape.batch, self.shape.h_q, self.shape.h_kv, self.shape.head_dim,
+                          self.shape.t_ctx - self.window, self.shape.t_cap)
+        if out is None:
+            out = torch.empty(self.shape.batch, self.shape.h_q, self.window, dtype=torch.float32,
+                              device=k_cache.device)
+        ws = B.Workspace(B.bd_workspace_size(sh, B.BD_OP_VERIFY, 1, self.window), k_cache.device)
+        B.bd_verify_attn(sh, q_win, self.window, k_cache, None, None, out, ws, stream)
+        return out

@@ -1,0 +1,123 @@
+"""Host-side checks of the C ABI (no GPU): the library builds and loads, exports every
+entry point include/budgetdraft.h declares, and rejects bad arguments before any
+launch.  Only validation paths are exercised: no pointer is dereferenced."""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2606_00144_gb300 as bd
+from paper_2606_00144_gb300 import binding
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(__file__)), "include", "budgetdraft.h")
+
+BD_OK, INVALID, UNSUPPORTED, MISALIGNED, WORKSPACE, CUDA_ERR, TIMEOUT = 0, -1, -2, -3, -4, -5, -6
+A = 0x10000          # a fake, 16-byte aligned address: validation never dereferences it
+
+
+@pytest.fixture(scope="module")
+def lib():
+    bd.build()
+    return bd.library()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(bd_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_four_hot_path_calls():
+    names = declared_functions()
+    for n in ("bd_select_budget", "bd_draft_attn", "bd_verify_attn", "bd_combine"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert sorted(binding.exported_symbols()) == declared_functions()
+
+
+def test_strerror(lib):
+    for code in (BD_OK, INVALID, UNSUPPORTED, MISALIGNED, WORKSPACE, CUDA_ERR, TIMEOUT):
+        assert bd.bd_strerror(code) not in ("", "unknown status")
+    assert bd.bd_strerror(12345) == "unknown status"
+
+
+def shape(**kw):
+    base = dict(batch=2, h_q=8, h_kv=2, head_dim=128, t_ctx=100, t_cap=110)
+    base.update(kw)
+    return bd.make_shape(**base)
+
+
+def verify(lib, s, q=A, n_q=6, k=A, v=A, o=A, lse=A, ws=A, nbytes=1 << 20):
+    return lib.bd_verify_attn(ctypes.byref(s) if s is not None else None, q, n_q, k, v, o, lse, ws, nbytes, None)
+
+
+def draft(lib, s, q=A, k=A, v=A, idx=A, cnt=A, budget=32, j=0, o=A, lse=A, ws=A, nbytes=1 << 20):
+    return lib.bd_draft_attn(ctypes.byref(s), q, k, v, idx, cnt, budget, j, o, lse, ws, nbytes, None)
+
+
+def select(lib, s, k=A, qw=A, lse=A, window=32, budget=40, sink=4, recent=8, chunk=1, idx=A, cnt=A, ws=A,
+           nbytes=1 << 20):
+    return lib.bd_select_budget(ctypes.byref(s), k, qw, lse, window, budget, sink, recent, chunk, idx, cnt, ws,
+                                nbytes, None)
+
+
+def test_verify_validation(lib):
+    assert verify(lib, None) == INVALID
+    assert verify(lib, shape(head_dim=96)) == UNSUPPORTED
+    assert verify(lib, shape(h_q=6, h_kv=4)) == INVALID             # h_q % h_kv != 0
+    assert verify(lib, shape(t_cap=50)) == INVALID                    # t_cap < t_ctx
+    assert verify(lib, shape(), q=0) == INVALID
+    assert verify(lib, shape(), k=A + 8) == MISALIGNED
+    assert verify(lib, shape(), o=A + 2) == MISALIGNED
+    assert verify(lib, shape(), n_q=0) == INVALID
+    assert verify(lib, shape(), n_q=11) == INVALID                    # t_ctx + n_q > t_cap
+    assert verify(lib, shape(), o=0, lse=0) == INVALID                # nothing to write
+    assert verify(lib, shape(t_cap=200), n_q=25) == UNSUPPORTED       # 4 * 25 rows > 96 with V
+    assert verify(lib, shape(t_cap=200), n_q=33, o=0) == UNSUPPORTED  # 4 * 33 rows > 128, lse only
+
+
+def test_draft_validation(lib):
+    assert draft(lib, shape(), idx=0) == INVALID
+    assert draft(lib, shape(), cnt=A + 2) == MISALIGNED
+    assert draft(lib, shape(), j=-1) == INVALID
+    assert draft(lib, shape(), j=10) == INVALID                       # t_ctx + j >= t_cap
+    assert draft(lib, shape(), budget=0) == INVALID
+    assert draft(lib, shape(h_q=6, h_kv=2)) == UNSUPPORTED            # group of 3
+
+
+def test_select_validation(lib):
+    assert select(lib, shape(), window=0) == INVALID
+    assert select(lib, shape(), window=101) == INVALID                # window > t_ctx
+    assert select(lib, shape(), budget=10, sink=4, recent=8) == INVALID   # sink + recent > budget
+    assert select(lib, shape(), chunk=0) == INVALID
+    assert select(lib, shape(), sink=-1) == INVALID
+    assert select(lib, shape(), lse=A + 1) == MISALIGNED
+    assert select(lib, shape(h_q=16, h_kv=1), window=32) == UNSUPPORTED  # 512 window rows > 256
+    assert select(lib, shape(), qw=0) == INVALID
+
+
+def test_combine_validation(lib):
+    f = lib.bd_combine
+    assert f(A, A, 0, 4, 128, A, A, None) == INVALID
+    assert f(A, A, 2, -1, 128, A, A, None) == INVALID
+    assert f(A, A, 2, 4, 32, A, A, None) == UNSUPPORTED
+    assert f(A, A, 2, 0, 128, A, A, None) == BD_OK                     # empty: no-op
+    assert f(A + 4, A, 2, 4, 128, A, A, None) == MISALIGNED
+    assert f(A, A, 2, 4, 128, 0, A, None) == INVALID
+
+
+def test_workspace_status_null(lib):
+    assert lib.bd_workspace_status(None, None) == INVALID
+
+
+def test_product_path_fails_loudly_without_library(monkeypatch, tmp_path):
+    monkeypatch.setattr(binding, "_lib", None)
+    monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError):
+        binding.library()

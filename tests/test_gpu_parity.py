@@ -1,0 +1,312 @@
+"""Parity of the CUDA path (through the C ABI) with the fp64 oracle on the same seeded inputs.
+
+Covers the five evaluation workloads (the 32-layer stack on whole and sampled layers), the
+16K budget sweep including the B >= T case, ragged shapes that span several tiles with a
+partial tail, the degenerate cases, the standalone merge and determinism.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import paper_2606_00144_gb300 as bd
+from paper_2606_00144_gb300 import workload as W
+from tests.parity import check_attention, check_selection, f64
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="session", autouse=True)
+def built():
+    bd.build()
+    bd.library()
+
+
+def host(inp):
+    return dict(K=f64(inp.k_cache), V=f64(inp.v_cache), QW=f64(inp.q_win), QD=f64(inp.q_draft),
+                QV=f64(inp.q_verify))
+
+
+def run_and_check(wl, inp, h, budgets=None, modes=("carry", "self"), chunk=1, check_steps=True, tag=""):
+    """Runs selection (both modes), gamma drafts on the oracle's selection, and verify."""
+    t = wl.t_ctx
+    lse_ref = oracle.window_lse(h["QW"], h["K"], t)
+    score_ref = oracle.window_scores(h["QW"], h["K"], lse_ref, t)
+    lse_dev = torch.from_numpy(lse_ref).float().cuda()
+    stats = {}
+    budgets = budgets or [wl.budget]
+    for budget in budgets:
+        n_recent = wl.n_recent if budget == wl.budget else budget // 4
+        st = bd.SpecStep.for_workload(wl, budget=budget, n_recent=n_recent, chunk=chunk)
+        idx_ref = np.full((wl.batch, wl.h_kv, budget), -1)
+        cnt_ref = np.zeros((wl.batch, wl.h_kv), dtype=np.int64)
+        for b in range(wl.batch):
+            for kv in range(wl.h_kv):
+                keep = oracle.select_from_scores(score_ref[b, kv], t, budget, wl.n_sink, n_recent, chunk)
+                idx_ref[b, kv, : keep.size] = keep
+                cnt_ref[b, kv] = keep.size
+        for mode in modes:
+            st.select(inp.k_cache, inp.q_win, lse_dev if mode == "carry" else None)
+            torch.cuda.synchronize()
+            nd = check_selection(st.idx, st.count, idx_ref, cnt_ref, score_ref, t, budget, wl.n_sink, n_recent,
+                                 chunk, what=f"{tag} B={budget} {mode}")
+            stats[f"select_B{budget}_{mode}_diff"] = nd
+        if not check_steps:
+            continue
+        # drafts on the oracle's selection (both sides see the same sparse view)
+        st.idx.copy_(torch.from_numpy(idx_ref).int())
+        st.count.copy_(torch.from_numpy(cnt_ref).int())
+        for j in range(wl.gamma):
+            st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
+            o_ref, l_ref = oracle.draft_attn(h["QD"][j], h["K"], h["V"], idx_ref, cnt_ref, t, j)
+            torch.cuda.synchronize()
+            stats[f"draft{j}_B{budget}"] = check_attention(st.draft_o[j], st.draft_lse[j], o_ref, l_ref,
+                                                           f"{tag} draft j={j} B={budget}")
+        if budget == budgets[0]:
+            st.verify(inp.q_verify, inp.k_cache, inp.v_cache)
+            o_ref, l_ref = oracle.verify_attn(h["QV"], h["K"], h["V"], t)
+            torch.cuda.synchronize()
+            stats["verify"] = check_attention(st.verify_o, st.verify_lse, o_ref, l_ref, f"{tag} verify")
+        assert st.ws.status() == 0
+    return stats
+
+
+# ----------------------------------------------------------------------------- evaluation workloads
+
+def test_tiny_1k():
+    wl = W.WORKLOADS["tiny_1k"]
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), tag="tiny_1k")
+
+
+def test_l8b_4k():
+    wl = W.WORKLOADS["l8b_4k"]
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), tag="l8b_4k")
+
+
+def test_l8b_8k_b4():
+    wl = W.WORKLOADS["l8b_8k_b4"]
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), tag="l8b_8k_b4")
+
+
+def test_l8b_16k_b8_budget_sweep():
+    wl = W.WORKLOADS["l8b_16k_b8"]
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), budgets=list(W.SWEEP_16K), modes=("carry",), tag="l8b_16k_b8")
+
+
+def test_l8b_16k_b8_self_mode_selection():
+    wl = W.WORKLOADS["l8b_16k_b8"]
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), modes=("self",), check_steps=False, tag="l8b_16k_b8")
+
+
+def test_full_budget_draft_equals_full_attention():
+    # B >= T: the sparse view is the whole prefix, so draft pass j equals full causal attention
+    wl = W.WORKLOADS["l8b_16k_b8"]
+    inp = W.make_layer(wl, 0, "cuda")
+    st = bd.SpecStep.for_workload(wl, budget=16384, n_recent=4096)
+    st.select(inp.k_cache, inp.q_win, None)
+    torch.cuda.synchronize()
+    assert (st.count == wl.t_ctx).all()
+    assert torch.equal(st.idx[..., : wl.t_ctx].cpu(), torch.arange(wl.t_ctx).expand(wl.batch, wl.h_kv, -1).int())
+    K, V = f64(inp.k_cache), f64(inp.v_cache)
+    for j in (0, wl.gamma - 1):
+        st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
+        q_blk = np.zeros((wl.batch, wl.h_q, j + 1, wl.head_dim))
+        q_blk[:, :, j] = f64(inp.q_draft[j])
+        o_ref, l_ref = oracle.verify_attn(q_blk, K, V, wl.t_ctx)
+        torch.cuda.synchronize()
+        check_attention(st.draft_o[j], st.draft_lse[j], o_ref[:, :, j], l_ref[:, :, j], f"full-budget draft {j}")
+
+
+def _unit_slice(inp, b, kv, group):
+    hs = slice(kv * group, (kv + 1) * group)
+    return dict(K=f64(inp.k_cache[b:b + 1, kv:kv + 1]), V=f64(inp.v_cache[b:b + 1, kv:kv + 1]),
+                QW=f64(inp.q_win[b:b + 1, hs]), QD=f64(inp.q_draft[:, b:b + 1, hs]),
+                QV=f64(inp.q_verify[b:b + 1, hs]))
+
+
+@pytest.mark.slow
+@pytest.mark.parametrize("layer,units", [(0, "all"), (31, [(0, 0), (7, 3), (15, 7)])])
+def test_l8b_32L_16k_b16_layers(layer, units):
+    wl = W.WORKLOADS["l8b_32L_16k_b16"]
+    inp = W.make_layer(wl, layer, "cuda")
+    st = bd.SpecStep.for_workload(wl)
+    lse_dev = st.window_lse(inp.k_cache, inp.q_win)     # carry state as a previous verify leaves it
+    st.run(inp.k_cache, inp.v_cache, inp.q_win, inp.q_draft, inp.q_verify, window_lse=lse_dev)
+    torch.cuda.synchronize()
+    if units == "all":
+        units = [(b, kv) for b in range(wl.batch) for kv in range(wl.h_kv)]
+    g, t = wl.group, wl.t_ctx
+    for b, kv in units:
+        h = _unit_slice(inp, b, kv, g)
+        lse_ref = oracle.window_lse(h["QW"], h["K"], t)
+        lse_gpu = f64(lse_dev[b, kv * g:(kv + 1) * g]).reshape(-1)
+        assert np.abs(lse_gpu - lse_ref.reshape(-1)).max() <= 1e-3
+        score = oracle.window_scores(h["QW"], h["K"], lse_ref, t)
+        keep = oracle.select_from_scores(score[0, 0], t, wl.budget, wl.n_sink, wl.n_recent)
+        idx_ref = np.full((1, 1, wl.budget), -1)
+        idx_ref[0, 0, : keep.size] = keep
+        check_selection(st.idx[b, kv], st.count[b, kv], idx_ref, np.array([keep.size]), score, t, wl.budget,
+                        wl.n_sink, wl.n_recent, what=f"32L layer {layer} ({b},{kv})")
+        vo, vl = oracle.verify_attn(h["QV"], h["K"], h["V"], t)
+        check_attention(st.verify_o[b, kv * g:(kv + 1) * g], st.verify_lse[b, kv * g:(kv + 1) * g], vo, vl,
+                        f"32L verify ({b},{kv})")
+        # drafts ran on the GPU's selection; compare where it equals the oracle's (else ties decided it)
+        gsel = st.idx[b, kv, : int(st.count[b, kv])].cpu().numpy()
+        if np.array_equal(gsel, keep):
+            for j in (0, wl.gamma - 1):
+                do, dl = oracle.draft_attn(h["QD"][j], h["K"], h["V"], idx_ref, np.array([[keep.size]]), t, j)
+                check_attention(st.draft_o[j, b, kv * g:(kv + 1) * g], st.draft_lse[j, b, kv * g:(kv + 1) * g],
+                                do, dl, f"32L draft {j} ({b},{kv})")
+    assert st.ws.status() == 0
+
+
+# ----------------------------------------------------------------------------- ragged and degenerate shapes
+
+RAGGED = [
+    # batch, h_q, h_kv, d, t_ctx, budget, sink, recent, window, gamma, chunk
+    (2, 8, 2, 128, 777, 100, 4, 20, 32, 5, 1),
+    (1, 4, 4, 64, 65, 16, 1, 3, 8, 3, 1),         # group 1, d 64, tail of one key
+    (3, 16, 2, 64, 333, 64, 0, 0, 16, 2, 1),      # group 8, no sink/recent
+    (1, 4, 1, 128, 1000, 200, 4, 8, 32, 5, 1),    # window wider than the recent set: causal scores
+    (2, 8, 2, 128, 640, 136, 0, 0, 32, 5, 8),     # the paper's chunk policy, s = 8
+    (1, 8, 2, 128, 1031, 128, 4, 32, 32, 5, 8),   # chunks with sink/recent and ragged chunk edges
+    (1, 8, 2, 128, 300, 36, 4, 32, 32, 1, 1),     # B = sink + recent: nothing ranked
+    (1, 8, 2, 64, 40, 64, 4, 8, 32, 5, 1),        # B > T
+]
+
+
+@pytest.mark.parametrize("case", RAGGED)
+def test_ragged_shapes(case):
+    b, hq, hkv, d, t, budget, sink, recent, window, gamma, chunk = case
+    wl = W.tiny_workload(batch=b, h_q=hq, h_kv=hkv, head_dim=d, t_ctx=t, budget=budget, n_sink=sink,
+                         n_recent=recent, window=window, gamma=gamma, seed=11 + t)
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), chunk=chunk, tag=f"ragged{case}")
+
+
+@pytest.mark.parametrize("n_q,with_v", [(1, True), (2, True), (12, True), (21, True), (32, False)])
+def test_verify_block_sizes(n_q, with_v):
+    wl = W.tiny_workload(batch=2, h_q=8, h_kv=2, head_dim=128, t_ctx=1500, gamma=n_q - 1 if n_q > 1 else 1)
+    inp = W.make_layer(wl, 0, "cuda")
+    q = torch.randn(wl.batch, wl.h_q, n_q, wl.head_dim, device="cuda").to(torch.bfloat16)
+    shape = bd.shape_of(inp.k_cache, wl.h_q, wl.t_ctx)
+    ws = bd.Workspace(bd.bd_workspace_size(shape, bd.BD_OP_VERIFY, 1, n_q))
+    o = torch.empty(wl.batch, wl.h_q, n_q, wl.head_dim, dtype=torch.bfloat16, device="cuda") if with_v else None
+    lse = torch.empty(wl.batch, wl.h_q, n_q, device="cuda")
+    bd.bd_verify_attn(shape, q, n_q, inp.k_cache, inp.v_cache, o, lse, ws)
+    o_ref, l_ref = oracle.verify_attn(f64(q), f64(inp.k_cache), f64(inp.v_cache), wl.t_ctx)
+    torch.cuda.synchronize()
+    if with_v:
+        check_attention(o, lse, o_ref, l_ref, f"verify n_q={n_q}")
+    else:
+        assert np.abs(f64(lse) - l_ref).max() <= 1e-3
+
+
+def test_draft_empty_view_and_full_view():
+    wl = W.tiny_workload(batch=2, h_q=8, h_kv=2, head_dim=128, t_ctx=500, budget=64)
+    inp = W.make_layer(wl, 0, "cuda")
+    h = host(inp)
+    st = bd.SpecStep.for_workload(wl)
+    rng = np.random.default_rng(3)
+    idx = np.full((2, 2, 64), -1)
+    cnt = np.array([[0, 64], [17, 1]])
+    for b in range(2):
+        for kv in range(2):
+            idx[b, kv, : cnt[b, kv]] = np.sort(rng.choice(500, cnt[b, kv], replace=False))
+    st.idx.copy_(torch.from_numpy(idx).int())
+    st.count.copy_(torch.from_numpy(cnt).int())
+    for j in range(wl.gamma):
+        st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
+        o_ref, l_ref = oracle.draft_attn(h["QD"][j], h["K"], h["V"], idx, cnt, wl.t_ctx, j)
+        torch.cuda.synchronize()
+        check_attention(st.draft_o[j], st.draft_lse[j], o_ref, l_ref, f"draft edge j={j}")
+
+
+def test_draft_out_of_range_index_is_reported_and_masked():
+    wl = W.tiny_workload(batch=1, h_q=4, h_kv=1, head_dim=64, t_ctx=100, budget=8)
+    inp = W.make_layer(wl, 0, "cuda")
+    h = host(inp)
+    st = bd.SpecStep.for_workload(wl)
+    idx = np.array([[[0, 5, 9, 100000, 20, -1, -1, -1]]])
+    st.idx.copy_(torch.from_numpy(idx).int())
+    st.count.fill_(5)
+    st.draft(0, inp.q_draft[0], inp.k_cache, inp.v_cache)
+    torch.cuda.synchronize()
+    assert st.ws.status() == -1                             # BD_ERR_INVALID_ARG recorded on the device
+    good = np.array([[[0, 5, 9, 20]]])
+    o_ref, l_ref = oracle.draft_attn(h["QD"][0], h["K"], h["V"], good, np.array([[4]]), wl.t_ctx, 0)
+    check_attention(st.draft_o[0], st.draft_lse[0], o_ref, l_ref, "draft masked bad index")
+    assert st.ws.status() == 0                              # reading clears it
+
+
+def test_combine_standalone():
+    rng = np.random.default_rng(5)
+    for n_split, rows, d in [(1, 3, 64), (5, 37, 128), (40, 9, 128)]:
+        o_part = rng.standard_normal((n_split, rows, d)).astype(np.float32)
+        lse_part = (rng.standard_normal((n_split, rows)) * 3).astype(np.float32)
+        lse_part[rng.random((n_split, rows)) < 0.2] = -np.inf
+        lse_part[:, 0] = -np.inf                     # an all-empty row
+        o_dev = torch.from_numpy(o_part).cuda()
+        l_dev = torch.from_numpy(lse_part).cuda()
+        out = torch.empty(rows, d, dtype=torch.bfloat16, device="cuda")
+        lse = torch.empty(rows, device="cuda")
+        bd.bd_combine(o_dev, l_dev, n_split, rows, d, out, lse)
+        o_ref, l_ref = oracle.combine(o_part.astype(np.float64), lse_part.astype(np.float64))
+        torch.cuda.synchronize()
+        check_attention(out, lse, o_ref, l_ref, f"combine {n_split}x{rows}x{d}")
+
+
+def test_combine_merges_disjoint_draft_views():
+    # attention over idx split into two disjoint halves, merged by bd_combine == attention over all
+    wl = W.tiny_workload(batch=1, h_q=8, h_kv=2, head_dim=128, t_ctx=900, budget=128)
+    inp = W.make_layer(wl, 0, "cuda")
+    h = host(inp)
+    rng = np.random.default_rng(9)
+    full = np.stack([np.sort(rng.choice(900, 128, replace=False)) for _ in range(2)])[None]
+    st = bd.SpecStep.for_workload(wl)
+    parts_o, parts_l = [], []
+    for half in (slice(0, 64), slice(64, 128)):
+        sub = np.full((1, 2, 128), -1)
+        sub[..., :64] = full[..., half]
+        st.idx.copy_(torch.from_numpy(sub).int())
+        st.count.fill_(64)
+        st.draft(0, inp.q_draft[0], inp.k_cache, inp.v_cache)
+        torch.cuda.synchronize()
+        parts_o.append(st.draft_o[0].float().reshape(-1, 128).clone())
+        parts_l.append(st.draft_lse[0].reshape(-1).clone())
+    # the tail row t_ctx is in both parts: remove it from the second by merging against it once
+    o_part = torch.stack(parts_o)
+    l_part = torch.stack(parts_l)
+    out = torch.empty(8, 128, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(8, device="cuda")
+    bd.bd_combine(o_part, l_part, 2, 8, 128, out, lse)
+    rows0 = np.concatenate([full[0, :, :64], np.full((2, 1), 900)], axis=1)
+    rows1 = np.concatenate([full[0, :, 64:], np.full((2, 1), 900)], axis=1)
+    o_ref = np.zeros((8, 128))
+    l_ref = np.zeros(8)
+    for hh in range(8):
+        kv = hh // 4
+        rows = np.concatenate([rows0[kv], rows1[kv]])       # the tail row counted twice, like the parts
+        o_ref[hh], l_ref[hh] = oracle.attention(h["QD"][0, 0, hh], h["K"][0, kv, rows], h["V"][0, kv, rows],
+                                                1 / np.sqrt(128))
+    torch.cuda.synchronize()
+    check_attention(out, lse, o_ref, l_ref, "combine of draft parts")
+
+
+def test_determinism():
+    wl = W.WORKLOADS["l8b_4k"]
+    inp = W.make_layer(wl, 0, "cuda")
+    outs = []
+    for _ in range(2):
+        st = bd.SpecStep.for_workload(wl)
+        st.run(inp.k_cache, inp.v_cache, inp.q_win, inp.q_draft, inp.q_verify)
+        torch.cuda.synchronize()
+        outs.append([t.clone() for t in (st.idx, st.count, st.draft_o, st.draft_lse, st.verify_o, st.verify_lse)])
+    for a, b in zip(*outs):
+        assert torch.equal(a, b)
