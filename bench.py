@@ -1,0 +1,571 @@
+#!/usr/bin/env python3
+"""Benchmark of one speculative step's KV-cache attention (BudgetDraft, Algorithm 2) on GB300.
+
+A step = KV-budget selection + gamma drafter decode passes over the sparse view + the
+verifier's (gamma+1)-query block pass, for every layer of the workload, through the C ABI.
+Default workload: Llama-3-8B-shaped layer, batch 8, 16K context, B = 512 (4 sink, 128
+recent), gamma = 5, window 32, selection with the carried window LSE.
+
+Prints ONE JSON line.  value = algorithmic HBM bytes of all ranks' steps / max-over-ranks
+time (GB/s); us_per_step and the per-kernel breakdown come from CUDA events on the
+launching stream inside the timed region.  The step is captured in a CUDA graph; inputs
+(K+V 537 MB at the default workload) exceed the 129 MB L2, so L2 is not flushed.
+
+  python bench.py [--config l8b_16k_b8] [--budget 512] [--sel-mode carry|self]
+                  [--steps K] [--warmup W] [--gpus N] [--impl reference]
+"""
+
+import os
+import sys
+
+if "OMP_NUM_THREADS" not in os.environ:           # the CPU baseline (numpy) uses every host core
+    _n = str(len(os.sched_getaffinity(0)))
+    for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        os.environ.setdefault(_v, _n)
+
+import argparse
+import ctypes
+import dataclasses
+import json
+import math
+import statistics
+import subprocess
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np
+import torch
+
+from paper_2606_00144_gb300 import workload as W
+
+METRIC = "spec-step attention µs & HBM GB/s (% of ~8 TB/s) at 16K ctx, B=512, γ=5"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+# ----------------------------------------------------------------------------- bytes the method must read
+
+def step_bytes(wl, budget, n_recent, sel_mode):
+    """Algorithmic HBM bytes of one step on one layer, by phase."""
+    row = wl.head_dim * 2
+    units = wl.batch * wl.h_kv
+    t = wl.t_ctx
+    if budget >= t:
+        sel = 0
+    else:
+        sel = (t - wl.n_sink - n_recent) * row * units          # middle keys, once
+        if sel_mode == "self":
+            sel += t * row * units                               # window LSE over the prefix
+    draft = (min(budget, t) + wl.gamma) * 2 * row * units       # sparse view once + drafted rows
+    verify = (t + wl.gamma + 1) * 2 * row * units
+    return dict(select=sel, draft=draft, verify=verify, total=sel + draft + verify)
+
+
+# ----------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+    NAMES = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+
+    def __init__(self, device):
+        self.proc = None
+        self.lines = []
+        try:
+            uuid = str(torch.cuda.get_device_properties(device).uuid)
+            self.sel = uuid if uuid.startswith("GPU-") else "GPU-" + uuid
+        except Exception:
+            self.sel = str(device)
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", self.sel, f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.1)
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        for ln in out.strip().splitlines():
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for name, val in zip(self.NAMES, parts[3:7]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        loaded = sorted(sm)[len(sm) // 2:] or sm                # samples under load (upper half)
+        return {"sm_mhz": statistics.median(loaded), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- distributed helpers
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ----------------------------------------------------------------------------- events inside graphs
+
+def timing_event():
+    try:
+        return torch.cuda.Event(enable_timing=True, external=True), None
+    except TypeError:       # older torch: record through the driver with the external flag
+        ev = torch.cuda.Event(enable_timing=True)
+        ev.record()
+        return ev, ctypes.CDLL("libcuda.so.1")
+
+
+def record(ev_pair):
+    ev, drv = ev_pair
+    if drv is None:
+        ev.record()
+    else:
+        drv.cuEventRecordWithFlags(ctypes.c_void_p(ev.cuda_event),
+                                   ctypes.c_void_p(torch.cuda.current_stream().cuda_stream), ctypes.c_uint(1))
+
+
+# ----------------------------------------------------------------------------- the GPU arm
+
+class Step:
+    """All layers of one workload: inputs, carried window LSE, one SpecStep per layer."""
+
+    def __init__(self, wl, budget, n_recent, sel_mode, device):
+        import paper_2606_00144_gb300 as bd
+        self.wl, self.budget, self.n_recent, self.sel_mode = wl, budget, n_recent, sel_mode
+        self.layers = [W.make_layer(wl, l, device) for l in range(wl.layers)]
+        self.steps = [bd.SpecStep.for_workload(wl, budget=budget, n_recent=n_recent, device=device)
+                      for _ in range(wl.layers)]
+        self.lse = []
+        for st, inp in zip(self.steps, self.layers):
+            # carried state: the window rows' LSE as the verify kernel leaves it
+            self.lse.append(st.window_lse(inp.k_cache, inp.q_win) if sel_mode == "carry" else None)
+        torch.cuda.synchronize()
+
+    def launches_per_step(self):
+        # selection: top-B only (B >= T), else score + top-B (+ the window-LSE pass in self mode)
+        if self.budget >= self.wl.t_ctx:
+            sel = 1
+        else:
+            sel = 2 + (1 if self.sel_mode == "self" else 0)
+        return self.wl.layers * (sel + self.wl.gamma + 1)
+
+    def run(self, marks=None):
+        """One step; marks = [select, draft, verify, end] timing events (or None)."""
+        L = range(self.wl.layers)
+        if marks:
+            record(marks[0])
+        for l in L:
+            self.steps[l].select(self.layers[l].k_cache, self.layers[l].q_win, self.lse[l])
+        if marks:
+            record(marks[1])
+        for j in range(self.wl.gamma):
+            for l in L:
+                inp = self.layers[l]
+                self.steps[l].draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
+        if marks:
+            record(marks[2])
+        for l in L:
+            inp = self.layers[l]
+            self.steps[l].verify(inp.q_verify, inp.k_cache, inp.v_cache)
+        if marks:
+            record(marks[3])
+
+
+class HostIO:
+    """Pinned host copies of one step's inputs and outputs for the end-to-end measurement.
+
+    Per step and layer the host sends the queries (window, gamma draft passes, verify
+    block), the carried window LSE and the K/V rows of the gamma+1 block tokens, and reads
+    back the selection, the draft outputs and the verify outputs.  The KV cache itself is
+    state that stays resident in HBM."""
+
+    def __init__(self, step: Step):
+        wl = step.wl
+        self.step = step
+        self.h2d, self.d2h = [], []
+        g1 = wl.gamma + 1
+        for l, (st, inp) in enumerate(zip(step.steps, step.layers)):
+            dev_rows_k = torch.empty(wl.batch, wl.h_kv, g1, wl.head_dim, dtype=torch.bfloat16, device="cuda")
+            dev_rows_v = torch.empty_like(dev_rows_k)
+            dev_rows_k.copy_(inp.k_cache[:, :, wl.t_ctx: wl.t_ctx + g1])
+            dev_rows_v.copy_(inp.v_cache[:, :, wl.t_ctx: wl.t_ctx + g1])
+            ins = [inp.q_win, inp.q_draft, inp.q_verify, dev_rows_k, dev_rows_v]
+            if step.lse[l] is not None:
+                ins.append(step.lse[l])
+            for d in ins:
+                self.h2d.append((torch.empty(d.shape, dtype=d.dtype, pin_memory=True).copy_(d.cpu()), d))
+            for d in (st.idx, st.count, st.draft_o, st.draft_lse, st.verify_o, st.verify_lse):
+                self.d2h.append((d, torch.empty(d.shape, dtype=d.dtype, pin_memory=True)))
+            self.h2d.append(("rows", l, dev_rows_k, dev_rows_v))
+        self.bytes_in = sum(h.numel() * h.element_size() for h, *_ in self.h2d if isinstance(h, torch.Tensor))
+        self.bytes_out = sum(h.numel() * h.element_size() for _, h in self.d2h)
+
+    def run(self):
+        wl = self.step.wl
+        g1 = wl.gamma + 1
+        for item in self.h2d:
+            if item[0] == "rows":
+                _, l, rk, rv = item
+                inp = self.step.layers[l]
+                inp.k_cache[:, :, wl.t_ctx: wl.t_ctx + g1].copy_(rk)
+                inp.v_cache[:, :, wl.t_ctx: wl.t_ctx + g1].copy_(rv)
+            else:
+                h, d = item
+                d.copy_(h, non_blocking=True)
+        self.step.run()
+        for d, h in self.d2h:
+            h.copy_(d, non_blocking=True)
+
+
+def capture(fn, n):
+    g = torch.cuda.CUDAGraph()
+    s = torch.cuda.Stream()
+    s.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(s):
+        with torch.cuda.graph(g, stream=s):
+            for i in range(n):
+                fn(i)
+    torch.cuda.current_stream().wait_stream(s)
+    return g
+
+
+def timed_replays(graphs, world):
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for g in graphs:
+        g.replay()
+    t1.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    return t0.elapsed_time(t1)
+
+
+def graph_len(k, limit):
+    """Steps per captured graph: the largest divisor of k not above limit, so that the
+    timed region is a whole number of replays of one graph."""
+    for s in range(max(1, min(k, limit)), 0, -1):
+        if k % s == 0:
+            return s
+    return 1
+
+
+def gpu_arm(args):
+    world, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    wl = resolve_workload(args)
+    n_recent = wl.n_recent
+    budget = wl.budget
+    step = Step(wl, budget, n_recent, args.sel_mode, "cuda")
+    per = step_bytes(wl, budget, n_recent, args.sel_mode)
+    layer_bytes = {k: v * wl.layers for k, v in per.items()}
+
+    # eager warm-up (first calls set kernel attributes), then capture
+    step.run()
+    torch.cuda.synchronize()
+    S = graph_len(args.steps, args.graph_steps)
+    marks = [[timing_event() for _ in range(4)] for _ in range(S)]
+    g_main = capture(lambda i: step.run(marks[i]), S)
+    g_warm = capture(lambda i: step.run(), 1)
+    for _ in range(args.warmup):
+        g_warm.replay()
+    torch.cuda.synchronize()
+
+    sampler = ClockSampler(local)
+    sampler.start()
+    ms = timed_replays([g_main] * (args.steps // S), world)
+    clocks = sampler.stop()
+    ms = max_over_ranks(ms, world)
+    # per-phase durations: the S steps of the last replay inside the timed region
+    ph = {"select": [], "draft": [], "verify": []}
+    for i in range(S):
+        e = [m[0] for m in marks[i]]
+        ph["select"].append(e[0].elapsed_time(e[1]))
+        ph["draft"].append(e[1].elapsed_time(e[2]))
+        ph["verify"].append(e[2].elapsed_time(e[3]))
+    phase_us = {k: 1000.0 * statistics.fmean(v) for k, v in ph.items()}
+
+    ms_per_step = ms / args.steps
+    us = 1000.0 * ms_per_step
+    total_bytes = layer_bytes["total"] * args.steps * world
+    value = total_bytes / (ms / 1e3) / 1e9
+    peak, peak_src = measured_hbm_peak()
+    verify_launch_bytes = per["verify"]
+    verify_us = phase_us["verify"] / wl.layers
+    achieved = verify_launch_bytes / (verify_us * 1e-6) / 1e9
+    line = {
+        "metric": METRIC,
+        "value": round(value, 1),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(ms_per_step, 5),
+        "us_per_step": round(us, 2),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "accum": "f32",
+        "data": "synthetic (seeded N(0,1) Q/K/V with planted heavy-hitter keys; see workload.py)",
+        "config": {
+            "workload": wl.name, "layers": wl.layers, "batch": wl.batch, "h_q": wl.h_q, "h_kv": wl.h_kv,
+            "head_dim": wl.head_dim, "t_ctx": wl.t_ctx, "budget": budget, "n_sink": wl.n_sink,
+            "n_recent": n_recent, "window": wl.window, "gamma": wl.gamma, "sel_mode": args.sel_mode,
+            "parallelism": f"replicas x{world}", "graph_steps": S,
+            "l2": "not flushed: K+V inputs (%.0f MB per layer) exceed the 129 MB L2"
+                  % ((wl.t_cap * 2 * wl.head_dim * 2 * wl.batch * wl.h_kv) / 1e6),
+        },
+        "pct_of_8tbs": round(100.0 * value / world / NOMINAL_HBM_GBS, 1),
+        "pct_of_measured_hbm": round(100.0 * value / world / peak, 1),
+        "tokens_verified_per_s": round(wl.batch * (wl.gamma + 1) * world / (ms_per_step / 1e3), 1),
+        "algorithmic_bytes_per_step": layer_bytes,
+        "breakdown_us": {k: round(v, 2) for k, v in phase_us.items()},
+        "roofline": {
+            "kernel": "verify_kernel (bd_verify_attn)",
+            "bound": "hbm",
+            "achieved": round(achieved, 1),
+            "peak": peak,
+            "peak_source": peak_src,
+            "unit": "GB/s",
+            "frac": round(achieved / peak, 3),
+            "bytes_per_launch": verify_launch_bytes,
+            "traffic": None,
+        },
+        "gpu_launches": step.launches_per_step() * args.steps,
+        "clocks": clocks,
+    }
+    if not args.no_e2e:
+        line["e2e"] = e2e_measure(step, args, world, layer_bytes["total"])
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, budget, n_recent, args.sel_mode, budget_s=args.cpu_seconds)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+def e2e_measure(step, args, world, bytes_per_step):
+    io = HostIO(step)
+    torch.cuda.synchronize()
+    S = graph_len(args.steps, args.graph_steps)
+    g = capture(lambda i: io.run(), S)
+    g.replay()
+    torch.cuda.synchronize()
+    ms = timed_replays([g] * (args.steps // S), world)
+    ms = max_over_ranks(ms, world)
+    value = bytes_per_step * args.steps * world / (ms / 1e3) / 1e9
+    return {"value": round(value, 1), "unit": "GB/s", "us_per_step": round(1000.0 * ms / args.steps, 2),
+            "h2d_bytes_per_step": io.bytes_in, "d2h_bytes_per_step": io.bytes_out,
+            "api": "paper_2606_00144_gb300.SpecStep through the C ABI, pinned host buffers, one CUDA graph"}
+
+
+def measured_hbm_peak():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs, copy)"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+# ----------------------------------------------------------------------------- oracle timing
+
+class OraclePieces:
+    """The oracle's step, one (sequence, KV head) unit at a time, in pieces:
+    selection (carried LSE), the gamma draft passes, the verify block."""
+
+    def __init__(self, wl, budget, n_recent, sel_mode):
+        import oracle
+        self.oracle = oracle
+        self.wl, self.budget, self.n_recent, self.sel_mode = wl, budget, n_recent, sel_mode
+        self.row = wl.head_dim * 2
+        self.units = [(b, kv) for b in range(wl.batch) for kv in range(wl.h_kv)]
+        self.seq_cache = {}
+        self.next_unit = 0
+        self.queue = []
+
+    def _unit(self, b, kv):
+        if b not in self.seq_cache:
+            self.seq_cache.clear()
+            one = dataclasses.replace(self.wl, batch=1)
+            inp = W.make_layer(one, 0, "cpu", first_seq=b)      # sequence b's own seed
+            f = lambda t: t.to(torch.float64).numpy()
+            self.seq_cache[b] = tuple(map(f, (inp.k_cache, inp.v_cache, inp.q_win, inp.q_draft, inp.q_verify)))
+        K, V, QW, QD, QV = self.seq_cache[b]
+        g = self.wl.group
+        hs = slice(kv * g, (kv + 1) * g)
+        return dict(K=K[:, kv:kv + 1], V=V[:, kv:kv + 1], QW=QW[:, hs], QD=QD[:, :, hs], QV=QV[:, hs])
+
+    def _refill(self):
+        b, kv = self.units[self.next_unit % len(self.units)]
+        self.next_unit += 1
+        u = self._unit(b, kv)
+        o = self.oracle
+        wl = self.wl
+        lse = None if self.sel_mode == "self" else o.window_lse(u["QW"], u["K"], wl.t_ctx)   # carried state
+        state = {}
+        sel_bytes = 0 if self.budget >= wl.t_ctx else (wl.t_ctx - wl.n_sink - self.n_recent) * self.row
+        if self.sel_mode == "self" and self.budget < wl.t_ctx:
+            sel_bytes += wl.t_ctx * self.row
+
+        def select():
+            idx, cnt, _ = o.select_budget(u["QW"], u["K"], wl.t_ctx, self.budget, wl.n_sink, self.n_recent,
+                                          1, lse)
+            state["idx"], state["cnt"] = idx, cnt
+
+        draft_bytes = (min(self.budget, wl.t_ctx) + wl.gamma) * 2 * self.row / wl.gamma
+
+        def draft(j):
+            return lambda: o.draft_attn(u["QD"][j], u["K"], u["V"], state["idx"], state["cnt"], wl.t_ctx, j)
+
+        def verify():
+            o.verify_attn(u["QV"], u["K"], u["V"], wl.t_ctx)
+
+        self.queue = [(select, sel_bytes)] + [(draft(j), draft_bytes) for j in range(wl.gamma)] + \
+                     [(verify, (wl.t_ctx + wl.gamma + 1) * 2 * self.row)]
+
+    def run_piece(self):
+        if not self.queue:
+            self._refill()
+        fn, nbytes = self.queue.pop(0)
+        t0 = time.perf_counter()
+        fn()
+        return time.perf_counter() - t0, nbytes
+
+
+def cpu_baseline(wl, budget, n_recent, sel_mode, budget_s=12.0):
+    pieces = OraclePieces(wl, budget, n_recent, sel_mode)
+    secs, nbytes, n = 0.0, 0.0, 0
+    per_unit = 2 + wl.gamma
+    t_start = time.perf_counter()
+    while (secs < budget_s or n % per_unit) and time.perf_counter() - t_start < 4 * budget_s:
+        s, b = pieces.run_piece()
+        secs += s
+        nbytes += b
+        n += 1
+    units = n // per_unit
+    return {"value": round(nbytes / secs / 1e9, 4), "unit": "GB/s",
+            "cores": int(os.environ.get("OMP_NUM_THREADS", "1")), "kind": "oracle",
+            "sample": f"{units} of {wl.batch * wl.h_kv} (sequence, KV head) units of one layer, full step "
+                      f"(selection with carried LSE, {wl.gamma} drafts, verify), numpy fp64; "
+                      f"{secs:.1f} s of oracle time"}
+
+
+def reference_arm(args):
+    world, rank, local = dist_env()
+    if rank != 0:
+        return
+    wl = resolve_workload(args)
+    pieces = OraclePieces(wl, wl.budget, wl.n_recent, args.sel_mode)
+    for _ in range(args.warmup):
+        pieces.run_piece()
+    secs, nbytes = 0.0, 0.0
+    for _ in range(args.steps):
+        s, b = pieces.run_piece()
+        secs += s
+        nbytes += b
+    value = nbytes / secs / 1e9
+    ms_per_step = 1e3 * secs / args.steps
+    cores = int(os.environ.get("OMP_NUM_THREADS", "1"))
+    sample = (f"each step = one piece of one (sequence, KV head) unit's step (selection with carried LSE, one of "
+              f"{wl.gamma} draft passes, or the verify block), round robin; fp64 numpy oracle")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic (same recipe as the GPU arm, drawn on the host)",
+        "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "h_q": wl.h_q, "h_kv": wl.h_kv,
+                   "head_dim": wl.head_dim, "t_ctx": wl.t_ctx, "budget": wl.budget, "n_sink": wl.n_sink,
+                   "n_recent": wl.n_recent, "window": wl.window, "gamma": wl.gamma, "sel_mode": args.sel_mode},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ----------------------------------------------------------------------------- CLI
+
+def resolve_workload(args):
+    wl = W.WORKLOADS[args.config]
+    if args.budget is not None and args.budget != wl.budget:
+        wl = wl.with_budget(args.budget)
+    return wl
+
+
+def parse():
+    p = argparse.ArgumentParser(description=__doc__.split("\n")[0])
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=4000)
+    p.add_argument("--warmup", type=int, default=50)
+    p.add_argument("--impl", choices=["gb300", "reference"], default="gb300")
+    p.add_argument("--config", default="l8b_16k_b8", choices=sorted(W.WORKLOADS))
+    p.add_argument("--budget", type=int, default=None)
+    p.add_argument("--sel-mode", choices=["carry", "self"], default="carry")
+    p.add_argument("--graph-steps", type=int, default=100, help="steps captured per CUDA graph")
+    p.add_argument("--cpu-seconds", type=float, default=12.0)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    a = p.parse_args()
+    if a.warmup < 3:
+        p.error("--warmup must be >= 3")
+    return a
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        reference_arm(args)
+    else:
+        gpu_arm(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -101,9 +101,11 @@ class LayerInputs:
     hh_pos: list = field(default_factory=list)   # per (b, kv): planted positions
 
 
-def make_layer(wl: Workload, layer: int = 0, device="cpu", out: dict | None = None) -> LayerInputs:
-    """Draw one layer's inputs.  If ``out`` holds preallocated bf16 tensors
-    (keys k_cache, v_cache, q_win, q_draft, q_verify) they are filled in place."""
+def make_layer(wl: Workload, layer: int = 0, device="cpu", out: dict | None = None,
+               first_seq: int = 0) -> LayerInputs:
+    """Draw one layer's inputs for sequences first_seq .. first_seq + batch - 1.  If
+    ``out`` holds preallocated bf16 tensors (keys k_cache, v_cache, q_win, q_draft,
+    q_verify) they are filled in place."""
     b, hq, hkv, d, tc = wl.batch, wl.h_q, wl.h_kv, wl.head_dim, wl.t_cap
     dev = torch.device(device)
     bf = torch.bfloat16
@@ -119,7 +121,7 @@ def make_layer(wl: Workload, layer: int = 0, device="cpu", out: dict | None = No
     n_hh = int(frac * wl.t_ctx)
     hh_pos = []
     for bi in range(b):
-        g = torch.Generator(device=dev).manual_seed(wl.seed + 1000 * layer + bi)
+        g = torch.Generator(device=dev).manual_seed(wl.seed + 1000 * layer + first_seq + bi)
         k = torch.randn(hkv, tc, d, generator=g, device=dev)
         v = torch.randn(hkv, tc, d, generator=g, device=dev)
         qw = torch.randn(hq, wl.window, d, generator=g, device=dev)
