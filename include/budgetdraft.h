@@ -128,6 +128,32 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
                   float* lse_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
+ * bd_draft_attn without a workspace.  The paper has no counterpart: this entry point
+ * exists for callers that cannot allocate device memory when they call the library,
+ * for example a plugin that is handed only a stream and tensor pointers by its host
+ * framework, or a serving loop whose device memory is fixed after start-up and which
+ * must not call cudaMalloc between steps.  Such callers cannot supply the workspace that
+ * bd_draft_attn needs.
+ *
+ * Arguments and results are those of bd_draft_attn, minus ws and ws_bytes.  The call
+ * allocates nothing: its scratch (status word, per-(sequence, KV head) counters and the
+ * split-K partials) is a 4 MiB array inside the library's device image, which every GPU
+ * that loads the library keeps until the process exits.  A shape whose scratch would not
+ * fit returns BD_ERR_WORKSPACE before any launch.
+ *   - The first call on a device looks up that array's device address with the device
+ *     current (cudaGetSymbolAddress); make that first call before any stream capture.
+ *   - Every call clears the array's status word and counters on `stream` before its
+ *     kernel.  Out-of-range indices are skipped as in bd_draft_attn, but this variant
+ *     does not report device-side errors.
+ *   - All calls share the one array: calls whose work can overlap on the GPU (different
+ *     streams, or threads without ordering between them) race and corrupt each other's
+ *     results.  Issue them on one stream.
+ */
+int bd_draft_attn_static(const bd_shape* shape, const void* q, const void* k_cache,
+                         const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
+                         int step_j, void* o_out, float* lse_out, void* stream);
+
+/*
  * Verifier block attention (Algorithm 2, Verify): query i (0 <= i < n_q) of head h
  * sits at position t_ctx + i and attends to keys [0, t_ctx + i] of its KV head.
  *   q        bf16 [batch, h_q, n_q, d]

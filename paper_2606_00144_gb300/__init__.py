@@ -15,6 +15,7 @@ from .binding import (  # noqa: F401
     Workspace,
     bd_combine,
     bd_draft_attn,
+    bd_draft_attn_static,
     bd_select_budget,
     bd_strerror,
     bd_verify_attn,

@@ -42,6 +42,8 @@ _SIGNATURES = {
                                         ctypes.c_int, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
     "bd_draft_attn": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P,
                                      ctypes.c_size_t, _P]),
+    "bd_draft_attn_static": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P,
+                                            _P]),
     "bd_verify_attn": (ctypes.c_int, [_SHAPE, _P, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "bd_combine": (ctypes.c_int, [_P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P, _P]),
     "bd_workspace_status": (ctypes.c_int, [_P, _P]),
@@ -144,6 +146,16 @@ def bd_draft_attn(shape, q, k_cache, v_cache, idx, count, budget, step_j, o_out,
                                  _ptr(count), int(budget), int(step_j), _ptr(o_out), _ptr(lse_out), ws.ptr,
                                  ws.nbytes, _stream(stream))
     _check("bd_draft_attn", st)
+
+
+def bd_draft_attn_static(shape, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out, stream=None):
+    """bd_draft_attn for callers that cannot allocate device memory: no workspace; the
+    library's own 4 MiB device array holds the scratch, shared by every call (calls must
+    not overlap on the GPU; the first call on a device must precede any stream capture)."""
+    st = library().bd_draft_attn_static(ctypes.byref(shape), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(idx),
+                                        _ptr(count), int(budget), int(step_j), _ptr(o_out), _ptr(lse_out),
+                                        _stream(stream))
+    _check("bd_draft_attn_static", st)
 
 
 def bd_verify_attn(shape, q, n_q, k_cache, v_cache, o_out, lse_out, ws: Workspace, stream=None):

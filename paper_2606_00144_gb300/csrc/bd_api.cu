@@ -178,6 +178,30 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
                                region(ws, units), counters(ws), status_word(ws), static_cast<cudaStream_t>(stream)));
 }
 
+// Allocation-free bd_draft_attn: the same validation and kernel, with the scratch taken
+// from the library's own device array (see bd_draft.cu) instead of a caller workspace.
+int bd_draft_attn_static(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
+                         const int32_t* idx, const int32_t* count, int budget, int step_j, void* o_out,
+                         float* lse_out, void* stream) {
+  BD_TRY(check_shape(shape));
+  const bd_shape& s = *shape;
+  BD_TRY(check_tensor(q, 16));
+  BD_TRY(check_tensor(k_cache, 16));
+  BD_TRY(check_tensor(v_cache, 16));
+  BD_TRY(check_tensor(idx, 4));
+  BD_TRY(check_tensor(count, 4));
+  BD_TRY(check_tensor(o_out, 16));
+  if (lse_out) BD_TRY(check_tensor(lse_out, 4));
+  if (budget < 1 || step_j < 0 || (long long)s.t_ctx + step_j >= s.t_cap) return BD_ERR_INVALID_ARG;
+  if (!group_supported_by_draft(s.h_q / s.h_kv)) return BD_ERR_UNSUPPORTED;
+  DraftPlan dp;
+  if (!draft_plan(s, budget, step_j + 1, &dp)) return BD_ERR_UNSUPPORTED;
+  const int units = s.batch * s.h_kv;
+  if (ws_region_offset(units) + draft_partials_bytes(s, dp) > draft_static_scratch_bytes()) return BD_ERR_WORKSPACE;
+  return map_cuda(launch_draft_static(s, dp, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
+                                      static_cast<cudaStream_t>(stream)));
+}
+
 int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_cache, const void* v_cache,
                    void* o_out, float* lse_out, void* ws, size_t ws_bytes, void* stream) {
   BD_TRY(check_shape(shape));

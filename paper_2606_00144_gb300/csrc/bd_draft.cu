@@ -9,6 +9,7 @@
 // with an online softmax.  Each CTA writes a normalised partial; the last CTA of a unit
 // merges them (log-sum-exp) into the bf16 output.
 #include <algorithm>
+#include <mutex>
 
 #include "bd_common.cuh"
 #include "bd_internal.h"
@@ -299,6 +300,57 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   DraftFn fn = pick(s.head_dim, s.h_q / s.h_kv);
   fn<<<dim3(plan.n_split, units), kDThreads, 0, stream>>>(p);
   return cudaGetLastError();
+}
+
+// ============================================================================ allocation-free variant
+//
+// bd_draft_attn_static runs the same kernel as bd_draft_attn, but its scratch (status
+// word, per-unit arrival counters, split partials) lives in this file-scope device array
+// instead of a caller-provided workspace, for callers that cannot allocate device memory.
+// The array is part of the library image: every GPU that loads the library holds it
+// until the process exits.  All calls share it, so calls that overlap on the GPU race.
+
+constexpr size_t kDraftStaticScratchBytes = size_t(4) << 20;   // 4 MiB
+static __device__ __align__(256) unsigned char g_draft_scratch[kDraftStaticScratchBytes];
+
+size_t draft_static_scratch_bytes() { return kDraftStaticScratchBytes; }
+
+// Device address of g_draft_scratch on the current device.  In host code the symbol is
+// only a host-side stand-in, so the address is looked up once per device, with that
+// device current, and cached.
+static cudaError_t draft_scratch_address(void** out) {
+  static std::mutex mu;
+  static void* addr[256] = {nullptr};
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  if (dev < 0 || dev >= 256) return cudaErrorInvalidDevice;
+  std::lock_guard<std::mutex> lock(mu);
+  if (addr[dev] == nullptr) {
+    void* p = nullptr;
+    err = cudaGetSymbolAddress(&p, g_draft_scratch);
+    if (err != cudaSuccess) return err;
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return cudaSuccess;
+}
+
+cudaError_t launch_draft_static(const bd_shape& s, const DraftPlan& plan, const void* q, const void* k_cache,
+                                const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
+                                int step_j, void* o_out, float* lse_out, cudaStream_t stream) {
+  void* base = nullptr;
+  cudaError_t err = draft_scratch_address(&base);
+  if (err != cudaSuccess) return err;
+  const int units = s.batch * s.h_kv;
+  uint8_t* b = static_cast<uint8_t*>(base);
+  // The array keeps whatever the previous call left: clear the status word and the
+  // arrival counters (they must start at zero) before this call's kernel.
+  err = cudaMemsetAsync(b, 0, ws_region_offset(units), stream);
+  if (err != cudaSuccess) return err;
+  return launch_draft(s, plan, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
+                      b + ws_region_offset(units), reinterpret_cast<int*>(b + ws_counters_offset()),
+                      reinterpret_cast<int*>(b), stream);
 }
 
 }  // namespace bd
