@@ -14,6 +14,8 @@ template <int D>
 __global__ void __launch_bounds__(kCThreads) combine_kernel(const float* o_part, const float* lse_part,
                                                             int n_split, int rows, int rows_per_block,
                                                             __nv_bfloat16* o_out, float* lse_out) {
+  grid_dependency_wait();
+  allow_dependent_launch();
   extern __shared__ float w_smem[];
   const int r0 = blockIdx.x * rows_per_block;
   const int nr = min(rows_per_block, rows - r0);
@@ -32,11 +34,9 @@ cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_spl
   const size_t smem = (size_t)n_split * rpb * sizeof(float);
   const dim3 grid((rows + rpb - 1) / rpb);
   __nv_bfloat16* o = static_cast<__nv_bfloat16*>(o_out);
-  if (head_dim == 64)
-    combine_kernel<64><<<grid, kCThreads, smem, stream>>>(o_part, lse_part, n_split, rows, rpb, o, lse_out);
-  else
-    combine_kernel<128><<<grid, kCThreads, smem, stream>>>(o_part, lse_part, n_split, rows, rpb, o, lse_out);
-  return cudaGetLastError();
+  void* args[] = {&o_part, &lse_part, &n_split, &rows, const_cast<int*>(&rpb), &o, &lse_out};
+  void* fn = head_dim == 64 ? reinterpret_cast<void*>(&combine_kernel<64>) : reinterpret_cast<void*>(&combine_kernel<128>);
+  return launch_kernel(fn, grid, dim3(kCThreads), smem, stream, args, 0);
 }
 
 }  // namespace bd

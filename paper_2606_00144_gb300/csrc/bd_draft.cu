@@ -1,23 +1,37 @@
 // Drafter decode pass over the sparse view (Algorithm 2, Draft): one query per head,
 // keys = the selected rows idx[0:count] plus the drafted rows t_ctx .. t_ctx+step_j.
 //
-// Memory-bound gather (4 flop per byte): the G query heads of a GQA group share every
-// gathered row, so one CTA serves one (sequence, KV head) unit and one slice of its entry
-// list.  Rows are gathered with 16-byte cp.async into padded shared-memory tiles (K
-// first, V behind it so its latency overlaps the QK^T), scores and softmax run in fp32 on
-// CUDA cores with warp-shuffle reductions, and a slice longer than one tile is folded in
-// with an online softmax.  Each CTA writes a normalised partial; the last CTA of a unit
-// merges them (log-sum-exp) into the bf16 output.
+// Memory-bound gather (4 flop per byte) whose cost is latency, so the design minimises
+// dependent round trips.  A thread-block cluster of up to 8 CTAs serves one (sequence,
+// KV head) unit, each CTA one slice of its entry list:
+//   1. count and the slice's indices are fetched together (indices speculatively, before
+//      count is known);
+//   2. rows are gathered with 16-byte cp.async straight into the 128-byte swizzled layout
+//      (unused rows zero-filled) and the four warps run the mma.sync sub-tile code shared
+//      with the verify kernel (bd_attn_warp.cuh), the G heads of the GQA group forming one
+//      n8 query tile;
+//   3. the CTAs' normalised partials are merged through distributed shared memory by the
+//      cluster's rank-0 CTA (log-sum-exp), which writes the bf16 output: no global
+//      partials, fences or atomics.
+// Launched with programmatic dependent launch: the grid-dependency wait is the first thing
+// a CTA does, and the next kernel may be scheduled as soon as every CTA has passed it.
+#include <cooperative_groups.h>
+
 #include <algorithm>
 #include <mutex>
 
+#include "bd_attn_warp.cuh"
 #include "bd_common.cuh"
 #include "bd_internal.h"
 
+namespace cg = cooperative_groups;
+
 namespace bd {
 
-constexpr int kDRows = 64;        // rows per shared-memory tile
-constexpr int kDThreads = 128;
+constexpr int kDRows = 80;        // rows per shared-memory tile (5 sub-tiles of 16)
+constexpr int kDSubs = kDRows / 16;
+constexpr int kDThreads = 128;    // 4 warps
+constexpr int kDMaxCluster = 8;   // portable cluster size
 
 struct DraftParams {
   const __nv_bfloat16* q;      // [units * G][D]
@@ -27,254 +41,228 @@ struct DraftParams {
   const int32_t* count;        // [units]
   __nv_bfloat16* o;            // [units * G][D]
   float* lse;                  // [units * G] or null
-  float* o_part;               // [n_split][units * G][D]
-  float* lse_part;             // [n_split][units * G]
-  int* counters;
   int* status;
-  int units, budget, step_j, t_ctx, t_cap, n_split, rows_per_split;
+  int budget, step_j, t_ctx, t_cap, n_split, rows_per_split;
+  int n_stage;                 // 1, or 2 when a CTA gathers more than one tile (double buffer)
   float scale_log2;
 };
 
 template <int D, int G>
+struct DraftSmem {
+  static constexpr uint32_t TILE_BYTES = kDRows * D * 2;
+  static constexpr uint32_t STAGE_BYTES = 2 * TILE_BYTES;                 // K and V
+  static constexpr size_t kMerge = (size_t)(3 * 4 * 8) * 4 + (size_t)4 * 8 * (D + 4) * 4;
+  // stages (the warp-merge scratch reuses them) | rowpos [2][kDRows] | partial o [G][D], lse [G]
+  static size_t bytes(int n_stage) {
+    const size_t stages = std::max<size_t>((size_t)n_stage * STAGE_BYTES, kMerge);
+    return 1024 + stages + 2 * kDRows * 4 + (size_t)G * D * 4 + G * 4 + 16;
+  }
+};
+
+template <int D, int G>
 __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
-  constexpr int PITCH = D + 8;                 // bf16 per tile row (16-byte pad: conflict-free)
-  constexpr int TPR = kDThreads / kDRows;      // threads per row in the score phase
-  constexpr int DP = D / 2;                    // bf16 pairs per row
-  constexpr int RG = kDThreads / DP;           // row groups in the PV phase
-  __shared__ __align__(16) __nv_bfloat16 ks[kDRows * PITCH];
-  __shared__ __align__(16) __nv_bfloat16 vs[kDRows * PITCH];
-  __shared__ float qf[G * D];
-  __shared__ float sc[kDRows * G];
-  __shared__ int rowpos[kDRows];
-  __shared__ float m_run[G], l_run[G], alpha_s[G];
-  __shared__ int last_flag;
+  using L = DraftSmem<D, G>;
+  constexpr uint32_t HALF_BYTES = kDRows * 128;
+  constexpr int CH = D / 8;                    // 16-byte chunks per row
+  grid_dependency_wait();
+  allow_dependent_launch();
+
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  constexpr size_t kMergeBytes = L::kMerge;
+  const size_t stage_bytes = (size_t)p.n_stage * L::STAGE_BYTES > kMergeBytes ? (size_t)p.n_stage * L::STAGE_BYTES
+                                                                               : kMergeBytes;
+  uint8_t* stage = smem;                                                  // n_stage x (K, V)
+  int* rowpos = reinterpret_cast<int*>(smem + stage_bytes);               // [2][kDRows]
+  float* part_o = reinterpret_cast<float*>(rowpos + 2 * kDRows);          // [G][D]
+  float* part_lse = part_o + G * D;                                       // [G]
+  float* m_s = reinterpret_cast<float*>(stage);                           // warp-merge scratch
+  float* l_s = m_s + 4 * 8;
+  float* f_s = l_s + 4 * 8;
+  float* o_s = f_s + 4 * 8;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int split = blockIdx.x, unit = blockIdx.y;
-  int cnt = p.count[unit];
+  const int32_t* iunit = p.idx + (size_t)unit * p.budget;
+  const int e_begin = split * p.rows_per_split;
+  // count and the first tile's indices in flight together
+  int idx_pref = -1;
+  if (tid < kDRows) {
+    const int e = e_begin + tid;
+    if (e < p.budget && tid < p.rows_per_split) idx_pref = __ldg(iunit + e);
+  }
+  int cnt = __ldg(p.count + unit);
   if (cnt < 0 || cnt > p.budget) {
     if (tid == 0) record_error(p.status, BD_ERR_INVALID_ARG);
     cnt = min(max(cnt, 0), p.budget);
   }
   const int n_entries = cnt + p.step_j + 1;
-  const int e_begin = split * p.rows_per_split;
   const int e_end = min(e_begin + p.rows_per_split, n_entries);
-
-  const __nv_bfloat16* qsrc = p.q + (size_t)unit * G * D;
-  for (int i = tid; i < G * D; i += kDThreads) qf[i] = __bfloat162float(qsrc[i]);
-  if (tid < G) {
-    m_run[tid] = -INFINITY;
-    l_run[tid] = 0.f;
-  }
+  const int n_tiles = e_end > e_begin ? (e_end - e_begin + kDRows - 1) / kDRows : 0;
   const __nv_bfloat16* kunit = p.k + (size_t)unit * p.t_cap * D;
   const __nv_bfloat16* vunit = p.v + (size_t)unit * p.t_cap * D;
-  const int32_t* iunit = p.idx + (size_t)unit * p.budget;
 
-  float acc[G][2];
-#pragma unroll
-  for (int g = 0; g < G; ++g) acc[g][0] = acc[g][1] = 0.f;
-  const int dp = tid % DP, rg = tid / DP;
-
-  for (int e0 = e_begin; e0 < e_end; e0 += kDRows) {
-    const int nrows = min(kDRows, e_end - e0);
-    __syncthreads();                           // previous tile fully consumed
-    if (tid < nrows) {
+  auto position = [&](int e, int idx_value) -> int {
+    if (e >= cnt) return p.t_ctx + (e - cnt);            // a drafted row
+    if (idx_value < 0 || idx_value >= p.t_ctx) {
+      record_error(p.status, BD_ERR_INVALID_ARG);
+      return -1;                                         // skipped
+    }
+    return idx_value;
+  };
+  // row positions of tile `tile` into rowpos[b] (threads < kDRows), then the gather
+  auto set_rows = [&](int tile, int b, bool prefetched) {
+    const int e0 = e_begin + tile * kDRows;
+    if (tid < kDRows) {
       const int e = e0 + tid;
-      int pos;
-      if (e < cnt) {
-        pos = __ldg(iunit + e);
-        if (pos < 0 || pos >= p.t_ctx) {
-          record_error(p.status, BD_ERR_INVALID_ARG);
-          pos = -1;
-        }
-      } else {
-        pos = p.t_ctx + (e - cnt);
-      }
-      rowpos[tid] = pos;
+      int pos = -1;
+      if (e < e_end) pos = position(e, prefetched ? idx_pref : (e < cnt ? __ldg(iunit + e) : 0));
+      rowpos[b * kDRows + tid] = pos;
     }
-    __syncthreads();
-    // gather K rows, then V rows (two cp.async groups)
-    for (int c = tid; c < nrows * (D / 8); c += kDThreads) {
-      const int r = c / (D / 8), ch = c % (D / 8);
-      const int pos = max(rowpos[r], 0);
-      cp_async16(ks + r * PITCH + ch * 8, kunit + (size_t)pos * D + ch * 8);
-    }
-    cp_async_commit();
-    for (int c = tid; c < nrows * (D / 8); c += kDThreads) {
-      const int r = c / (D / 8), ch = c % (D / 8);
-      const int pos = max(rowpos[r], 0);
-      cp_async16(vs + r * PITCH + ch * 8, vunit + (size_t)pos * D + ch * 8);
+  };
+  auto gather = [&](int tile, int b) {
+    const int nrows = min(kDRows, e_end - (e_begin + tile * kDRows));
+    uint8_t* kt = stage + b * L::STAGE_BYTES;
+    uint8_t* vt = kt + L::TILE_BYTES;
+    for (int c = tid; c < kDRows * CH; c += kDThreads) {
+      const int r = c / CH, ch = c % CH;
+      const uint32_t off = sw128_offset(r, ch * 8, HALF_BYTES);
+      const int pos = rowpos[b * kDRows + r];
+      const bool live = r < nrows && pos >= 0;   // others zero-filled (0 * garbage could be NaN in P V)
+      const size_t src = (size_t)max(pos, 0) * D + ch * 8;
+      cp_async16_zfill(kt + off, kunit + src, live);
+      cp_async16_zfill(vt + off, vunit + src, live);
     }
     cp_async_commit();
-    cp_async_wait<1>();
-    __syncthreads();
+  };
 
-    // scores: TPR threads per row, interleaved 16-byte chunks
-    {
-      const int r = tid / TPR, part = tid % TPR;
-      float s[G];
-#pragma unroll
-      for (int g = 0; g < G; ++g) s[g] = 0.f;
-#pragma unroll 4
-      for (int ch = part; ch < D / 8; ch += TPR) {
-        const uint4 raw = *reinterpret_cast<const uint4*>(ks + r * PITCH + ch * 8);
-        const __nv_bfloat162* kv2 = reinterpret_cast<const __nv_bfloat162*>(&raw);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const float2 kf = __bfloat1622float2(kv2[j]);
-#pragma unroll
-          for (int g = 0; g < G; ++g) {
-            s[g] = fmaf(qf[g * D + ch * 8 + 2 * j], kf.x, s[g]);
-            s[g] = fmaf(qf[g * D + ch * 8 + 2 * j + 1], kf.y, s[g]);
-          }
-        }
-      }
-#pragma unroll
-      for (int off = 1; off < TPR; off <<= 1)
-#pragma unroll
-        for (int g = 0; g < G; ++g) s[g] += __shfl_xor_sync(0xffffffffu, s[g], off);
-      if (part == 0) {
-        const bool ok = r < nrows && rowpos[r] >= 0;
-#pragma unroll
-        for (int g = 0; g < G; ++g) sc[r * G + g] = ok ? s[g] * p.scale_log2 : -INFINITY;
-      }
+  uint32_t bq[1][D / 16][2];
+  WarpAttn<D, 1, true>::load_q(bq, p.q + (size_t)unit * G * D, G, 0, lane);
+  WarpAttn<D, 1, true> wa;
+  wa.init();
+  const bool dbuf = p.n_stage == 2;
+  if (n_tiles > 0) {
+    set_rows(0, 0, true);
+    __syncthreads();
+    gather(0, 0);
+  }
+  for (int t = 0; t < n_tiles; ++t) {
+    const int b = dbuf ? (t & 1) : 0;
+    if (dbuf && t + 1 < n_tiles) {
+      set_rows(t + 1, (t + 1) & 1, false);
+      __syncthreads();
+      gather(t + 1, (t + 1) & 1);
+      cp_async_wait<1>();
+    } else {
+      cp_async_wait<0>();
     }
     __syncthreads();
-    // softmax bookkeeping per head (one warp per head, heads strided over the 4 warps)
-    for (int g = warp; g < G; g += kDThreads / 32) {
+    const int nrows = min(kDRows, e_end - (e_begin + t * kDRows));
+    const uint32_t kbase = smem_u32(stage + b * L::STAGE_BYTES);
+    const int* rp = rowpos + b * kDRows;
+    for (int sub = warp; sub < kDSubs && 16 * sub < nrows; sub += 4) {
+      const int kb = 16 * sub;
+      wa.step(kbase, kbase + L::TILE_BYTES, HALF_BYTES, kb, bq, p.scale_log2, lane, [&](int ko, int, int) {
+        const int r = kb + ko;
+        return r < nrows && rp[r] >= 0;
+      });
+    }
+    __syncthreads();                              // buffer b is free again
+    if (!dbuf && t + 1 < n_tiles) {
+      set_rows(t + 1, 0, false);
+      __syncthreads();
+      gather(t + 1, 0);
+    }
+  }
+  wa.finish_rows();
+  wa.store(m_s, l_s, o_s, warp, 8, 0, lane);
+  __syncthreads();
+  const size_t row0 = (size_t)unit * G;
+  if (p.n_split == 1) {
+    merge_warps_and_store<D, 4, true>(m_s, l_s, f_s, o_s, 8, G, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D, true,
+                                      tid, kDThreads, 0);
+    return;
+  }
+  merge_warps_and_store<D, 4, true>(m_s, l_s, f_s, o_s, 8, G, part_lse, part_o, false, tid, kDThreads, 0);
+
+  // ---------------------------------------------------------------- cluster merge (DSMEM)
+  cg::cluster_group cluster = cg::this_cluster();
+  cluster.sync();                                  // every CTA's partial is in its shared memory
+  if (cluster.block_rank() == 0) {
+    const int C = p.n_split;
+    float* wts = o_s;                              // [C][G] weights, then scale
+    if (tid < G) {
       float mx = -INFINITY;
-      for (int r = lane; r < kDRows; r += 32) mx = fmaxf(mx, sc[r * G + g]);
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
-      const float m_old = m_run[g];
-      const float m_new = fmaxf(m_old, mx);
-      const float m_use = m_new == -INFINITY ? 0.f : m_new;
-      float sum = 0.f;
-      for (int r = lane; r < kDRows; r += 32) {
-        const float pr = fast_exp2(sc[r * G + g] - m_use);
-        sc[r * G + g] = pr;
-        sum += pr;
+      for (int r = 0; r < C; ++r) mx = fmaxf(mx, *cluster.map_shared_rank(part_lse + tid, r));
+      float tot = 0.f;
+      for (int r = 0; r < C; ++r) {
+        const float l = *cluster.map_shared_rank(part_lse + tid, r);
+        const float w = mx == -INFINITY ? 0.f : fast_exp2((l - mx) * kLog2e);
+        wts[r * G + tid] = w;
+        tot += w;
       }
-#pragma unroll
-      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
-      __syncwarp();
-      if (lane == 0) {
-        const float al = fast_exp2(m_old - m_use);
-        alpha_s[g] = al;
-        l_run[g] = l_run[g] * al + sum;
-        m_run[g] = m_new;
-      }
+      const float inv = tot > 0.f ? 1.f / tot : 0.f;
+      for (int r = 0; r < C; ++r) wts[r * G + tid] *= inv;
+      if (p.lse) p.lse[row0 + tid] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
     }
-    cp_async_wait<0>();
     __syncthreads();
-    // O += P V (fp32), thread = (bf16 pair dp, row group rg)
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-      acc[g][0] *= alpha_s[g];
-      acc[g][1] *= alpha_s[g];
-    }
-    for (int r = rg; r < nrows; r += RG) {
-      const float2 vf = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(vs + r * PITCH + 2 * dp));
-#pragma unroll
-      for (int g = 0; g < G; ++g) {
-        const float pr = sc[r * G + g];
-        acc[g][0] = fmaf(pr, vf.x, acc[g][0]);
-        acc[g][1] = fmaf(pr, vf.y, acc[g][1]);
+    for (int i = tid; i < G * (D / 2); i += kDThreads) {
+      const int g = i / (D / 2), d = (i % (D / 2)) * 2;
+      float a0 = 0.f, a1 = 0.f;
+      for (int r = 0; r < C; ++r) {
+        const float w = wts[r * G + g];
+        const float2 v = *reinterpret_cast<const float2*>(cluster.map_shared_rank(part_o + g * D + d, r));
+        a0 += w * v.x;
+        a1 += w * v.y;
       }
+      *reinterpret_cast<uint32_t*>(p.o + (row0 + g) * D + d) = pack_bf16x2(a0, a1);
     }
   }
-
-  // reduce the row groups, normalise, write
-  __syncthreads();
-  float* red = reinterpret_cast<float*>(ks);   // [RG][G][D] floats (fits in the K tile)
-#pragma unroll
-  for (int g = 0; g < G; ++g) {
-    red[(rg * G + g) * D + 2 * dp] = acc[g][0];
-    red[(rg * G + g) * D + 2 * dp + 1] = acc[g][1];
-  }
-  __syncthreads();
-  const bool direct = p.n_split == 1;
-  for (int i = tid; i < G * D; i += kDThreads) {
-    const int g = i / D, d = i % D;
-    float a = 0.f;
-    for (int j = 0; j < RG; ++j) a += red[(j * G + g) * D + d];
-    const float l = l_run[g];
-    const float o = l > 0.f ? a / l : 0.f;
-    const size_t row = (size_t)unit * G + g;
-    if (direct) {
-      p.o[row * D + d] = __float2bfloat16_rn(o);
-    } else {
-      p.o_part[((size_t)split * p.units * G + row) * D + d] = o;
-    }
-  }
-  if (tid < G) {
-    const float l = l_run[tid];
-    const float lse = l > 0.f ? (m_run[tid] + log2f(l)) * kLn2 : -INFINITY;
-    const size_t row = (size_t)unit * G + tid;
-    if (direct) {
-      if (p.lse) p.lse[row] = lse;
-    } else {
-      p.lse_part[(size_t)split * p.units * G + row] = lse;
-    }
-  }
-  if (direct) return;
-
-  __threadfence();
-  __syncthreads();
-  if (tid == 0) last_flag = (atomicAdd(&p.counters[unit], 1) == p.n_split - 1);
-  __syncthreads();
-  if (last_flag) {
-    __threadfence();
-    const size_t row0 = (size_t)unit * G;
-    float* w = reinterpret_cast<float*>(vs);   // n_split * G floats
-    merge_partials<D>(p.o_part + row0 * D, p.lse_part + row0, p.n_split, G, (size_t)p.units * G * D,
-                      (size_t)p.units * G, p.o + row0 * D, p.lse ? p.lse + row0 : nullptr,
-                      [](int r) { return r; }, w, tid, kDThreads, 0);
-    if (tid == 0) p.counters[unit] = 0;
-  }
+  cluster.sync();                                  // partials stay alive until rank 0 has read them
 }
 
 // ============================================================================ host side
 
 namespace {
-using DraftFn = void (*)(DraftParams);
+using DraftFn = void*;
 DraftFn pick(int d, int g) {
 #define BD_DK(DD, GG) \
-  if (d == DD && g == GG) return &draft_kernel<DD, GG>;
+  if (d == DD && g == GG) return reinterpret_cast<void*>(&draft_kernel<DD, GG>);
   BD_DK(64, 1) BD_DK(64, 2) BD_DK(64, 4) BD_DK(64, 8)
   BD_DK(128, 1) BD_DK(128, 2) BD_DK(128, 4) BD_DK(128, 8)
 #undef BD_DK
   return nullptr;
 }
+size_t smem_bytes(int d, int g, int n_stage) {
+#define BD_DS(DD, GG) \
+  if (d == DD && g == GG) return DraftSmem<DD, GG>::bytes(n_stage);
+  BD_DS(64, 1) BD_DS(64, 2) BD_DS(64, 4) BD_DS(64, 8)
+  BD_DS(128, 1) BD_DS(128, 2) BD_DS(128, 4) BD_DS(128, 8)
+#undef BD_DS
+  return 0;
+}
 }  // namespace
-
-// The last CTA's merge weights (n_split * G floats) live in the V tile.
-static int max_split_for_merge(int d, int g) { return (kDRows * (d + 8) * 2) / (g * 4); }
 
 bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
   const int g = s.h_q / s.h_kv;
   if (!pick(s.head_dim, g)) return false;
-  const int units = s.batch * s.h_kv;
   const long entries = (long)budget + n_steps;
-  const int cap = std::max(1, 4 * current_sm_count() / std::max(1, units));
-  int n_split = (int)std::min<long>((entries + kDRows - 1) / kDRows, cap);
-  n_split = std::min(std::max(n_split, 1), max_split_for_merge(s.head_dim, g));
+  int n_split = (int)std::min<long>((entries + kDRows - 1) / kDRows, kDMaxCluster);
+  n_split = std::max(n_split, 1);
   plan->n_entries_max = (int)entries;
   plan->rows_per_split = (int)((entries + n_split - 1) / n_split);
-  plan->n_split = (int)((entries + plan->rows_per_split - 1) / plan->rows_per_split);
+  plan->n_split = n_split;
   return true;
 }
 
-size_t draft_partials_bytes(const bd_shape& s, const DraftPlan& plan) {
-  if (plan.n_split <= 1) return 0;
-  const size_t rows = (size_t)plan.n_split * s.batch * s.h_q;
-  return align_up(rows * s.head_dim * 4, 256) + align_up(rows * 4, 256);
-}
+size_t draft_partials_bytes(const bd_shape&, const DraftPlan&) { return 0; }   // merged in the cluster
 
 cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q, const void* k_cache,
                          const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
                          int step_j, void* o_out, float* lse_out, void* ws_region, int* counters,
                          int* status, cudaStream_t stream) {
+  (void)ws_region;
+  (void)counters;
   const int units = s.batch * s.h_kv;
   DraftParams p;
   p.q = static_cast<const __nv_bfloat16*>(q);
@@ -284,22 +272,23 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.count = count;
   p.o = static_cast<__nv_bfloat16*>(o_out);
   p.lse = lse_out;
-  const size_t rows = (size_t)plan.n_split * s.batch * s.h_q;
-  p.o_part = static_cast<float*>(ws_region);
-  p.lse_part = reinterpret_cast<float*>(static_cast<uint8_t*>(ws_region) + align_up(rows * s.head_dim * 4, 256));
-  p.counters = counters;
   p.status = status;
-  p.units = units;
   p.budget = budget;
   p.step_j = step_j;
   p.t_ctx = s.t_ctx;
   p.t_cap = s.t_cap;
   p.n_split = plan.n_split;
   p.rows_per_split = plan.rows_per_split;
+  p.n_stage = plan.rows_per_split > kDRows ? 2 : 1;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
-  DraftFn fn = pick(s.head_dim, s.h_q / s.h_kv);
-  fn<<<dim3(plan.n_split, units), kDThreads, 0, stream>>>(p);
-  return cudaGetLastError();
+  const int g = s.h_q / s.h_kv;
+  void* fn = pick(s.head_dim, g);
+  const size_t smem = smem_bytes(s.head_dim, g, p.n_stage);
+  cudaError_t err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  void* args[] = {&p};
+  return launch_kernel(fn, dim3(plan.n_split, units), dim3(kDThreads), smem, stream, args,
+                       plan.n_split > 1 ? plan.n_split : 0);
 }
 
 // ============================================================================ allocation-free variant

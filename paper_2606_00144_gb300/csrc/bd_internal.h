@@ -14,6 +14,12 @@ namespace bd {
 // ---------------------------------------------------------------------------- device facts
 int current_sm_count();   // SMs of the current device (cached per device)
 
+// Launch with programmatic dependent launch allowed (the kernel may be scheduled while
+// its predecessor finishes; every kernel of this library waits on the grid dependency
+// before touching its inputs) and, when cluster_x > 0, as clusters of cluster_x CTAs.
+cudaError_t launch_kernel(const void* fn, dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                          void** args, int cluster_x);
+
 // ---------------------------------------------------------------------------- workspace
 // [0, 256): status word; [256, 256 + units*4 rounded to 256): per-unit arrival counters;
 // then the op-specific region.
@@ -24,9 +30,11 @@ size_t ws_region_offset(int units);
 struct VerifyPlan {
   int nq_rows;          // query rows per (sequence, KV head) = group * n_q
   int nt, wq;           // n-tiles per warp, warp groups along queries
-  int n_tiles;          // 64-key tiles over [0, t_ctx + n_q)
-  int tiles_per_split;
-  int n_split;
+  int tiles_per_unit;   // 64-key tiles over [0, t_ctx + n_q)
+  int total_tiles;      // over all units
+  int tiles_per_cta;    // contiguous range of the global tile list per CTA
+  int grid;
+  int max_seg;          // most CTAs that share one unit
   int stages;
   size_t smem_bytes;
   bool with_v;
@@ -65,6 +73,7 @@ struct SelectPlan {
   int n_mid, n_mid_pad;
   int tiles_per_unit, total_tiles, grid, tiles_per_cta;
   int stages;
+  int n_acc;            // TMEM accumulators
   uint32_t tmem_cols;
   size_t smem_bytes;
   size_t score_bytes, lse_bytes;
@@ -89,5 +98,8 @@ int combine_rows_per_block(int n_split);
 // box_rows rows x 1 unit, 128-byte swizzle.
 cudaError_t make_cache_map(CUtensorMap* map, const void* base, int units, int t_cap, int n_rows,
                            int head_dim, int box_rows);
+// 2-D map over a dense [n_rows, head_dim] bf16 matrix; box = 64 columns x box_rows rows,
+// 128-byte swizzle; rows past n_rows read as zero.
+cudaError_t make_rows_map(CUtensorMap* map, const void* base, long long n_rows, int head_dim, int box_rows);
 
 }  // namespace bd

@@ -10,9 +10,11 @@
 //                 warp 1   one lane issues tcgen05.mma into a double-buffered fp32 TMEM
 //                          accumulator and commits to the smem/TMEM barriers;
 //                 warps 2-5 epilogue: tcgen05.ld, ex2 (MUFU), row sums, coalesced store.
-// topk_kernel   one CTA per (sequence, KV head): 4-pass MSB radix select on the fp32 score
-//               bits (warp-aggregated shared histograms), lower-index tie break by a block
-//               scan over the equal keys, ascending compaction with sinks and recents.
+// topk_kernel   one CTA per (sequence, KV head), scores staged in shared memory: a linear
+//               histogram between the min and max score finds the bin holding the k-th
+//               largest; that bin's few items are ranked exactly by (score desc, position
+//               asc) (4-pass radix select on the fp32 bits when the bin is crowded); then an
+//               ascending compaction (warp ballots + block scan) with sinks and recents.
 #include <algorithm>
 
 #include "bd_common.cuh"
@@ -21,8 +23,13 @@
 namespace bd {
 
 constexpr int kSKeys = 128;          // keys per tile (UMMA M)
-constexpr int kSThreads = 192;       // producer, MMA, 4 epilogue warps
+constexpr int kSThreads = 320;       // producer, MMA, 2 x 4 epilogue warps
+constexpr int kMaxAcc = 4;           // TMEM accumulators (<= 512 columns)
+constexpr int kSQOffset = 8192;      // shared-memory offset of the window-query tiles
 constexpr int kTopkThreads = 1024;
+constexpr int kTopkSmemBytes = 200 * 1024;   // item values staged in shared memory up to this size
+constexpr int kBins = 4096;                   // linear histogram bins of the value range
+constexpr int kBinCandMax = 2048;             // items of the boundary bin ranked exactly
 
 struct ScoreParams {
   const __nv_bfloat16* q_win;   // [units * nq_rows][D]
@@ -31,45 +38,50 @@ struct ScoreParams {
   int* status;
   int nq_rows, nq_pad, window, t_ctx, n_sink, mid_end, n_mid_pad;
   int tiles_per_unit, total_tiles, tiles_per_cta;
-  int acc_stride;               // TMEM columns between the two accumulators
+  int acc_stride;               // TMEM columns between accumulators
+  int n_acc;                    // accumulators: tile i uses i % n_acc; epilogue group i % 2
   uint32_t tmem_cols;
   float scale_log2;
 };
 
 template <int D, int STAGES>
 __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p,
-                                                             const __grid_constant__ CUtensorMap kmap) {
+                                                             const __grid_constant__ CUtensorMap kmap,
+                                                             const __grid_constant__ CUtensorMap qmap) {
   constexpr uint32_t KHALF = kSKeys * 128;         // one 64-column half of a K tile
   constexpr uint32_t KTILE = kSKeys * D * 2;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem);
   uint64_t* empty_bar = full_bar + STAGES;
-  uint64_t* tfull_bar = empty_bar + STAGES;
-  uint64_t* tempty_bar = tfull_bar + 2;
-  uint64_t* qfull_bar = tempty_bar + 2;
+  uint64_t* tfull_bar = empty_bar + STAGES;        // [kMaxAcc]
+  uint64_t* tempty_bar = tfull_bar + kMaxAcc;      // [kMaxAcc]
+  uint64_t* qfull_bar = tempty_bar + kMaxAcc;
   uint64_t* qempty_bar = qfull_bar + 2;
   uint64_t* drain_bar = qempty_bar + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* lse2_s = reinterpret_cast<float*>(smem + 1024);     // [288]
-  int* pw_s = reinterpret_cast<int*>(smem + 2304);            // [288]
   const uint32_t qbytes = (uint32_t)p.nq_pad * D * 2;
-  uint8_t* qbuf = smem + 4096;                                 // 2 x qbytes
+  uint8_t* qbuf = smem + kSQOffset;                            // 2 x qbytes
   uint8_t* kstage = qbuf + 2 * qbytes;                         // STAGES x KTILE (1024-aligned)
 
+  grid_dependency_wait();
+  allow_dependent_launch();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int first = blockIdx.x * p.tiles_per_cta;
   const int n = max(0, min(p.tiles_per_cta, p.total_tiles - first));
+  const int n_acc = p.n_acc;
 
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full_bar[s], 1);
       mbar_init(&empty_bar[s], 1);
     }
+    for (int a = 0; a < kMaxAcc; ++a) {
+      mbar_init(&tfull_bar[a], 1);
+      mbar_init(&tempty_bar[a], 4);
+    }
     for (int i = 0; i < 2; ++i) {
-      mbar_init(&tfull_bar[i], 1);
-      mbar_init(&tempty_bar[i], 4);
       mbar_init(&qfull_bar[i], 1);
       mbar_init(&qempty_bar[i], 1);
     }
@@ -88,7 +100,10 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
-    if (lane == 0) tma_prefetch_map(&kmap);
+    if (lane == 0) {
+      tma_prefetch_map(&kmap);
+      tma_prefetch_map(&qmap);
+    }
     int cur_unit = -1, qcount = 0;
     for (int i = 0; i < n; ++i) {
       const int g = first + i;
@@ -96,20 +111,19 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       if (unit != cur_unit) {
         const int qs = qcount & 1;
         bool ok = true;
-        if (qcount >= 2) ok = mbar_wait(&qempty_bar[qs], ((qcount >> 1) - 1) & 1, p.status, abort_flag);
-        if (!__all_sync(0xffffffffu, ok)) break;
-        uint8_t* qb = qbuf + qs * qbytes;
-        const __nv_bfloat16* src = p.q_win + (size_t)unit * p.nq_rows * D;
-        const uint32_t half_bytes = (uint32_t)p.nq_pad * 128;
-        for (int c = lane; c < p.nq_pad * (D / 8); c += 32) {
-          const int r = c / (D / 8), ch = c % (D / 8);
-          uint4 val = make_uint4(0u, 0u, 0u, 0u);
-          if (r < p.nq_rows) val = __ldg(reinterpret_cast<const uint4*>(src + (size_t)r * D + ch * 8));
-          *reinterpret_cast<uint4*>(qb + sw128_offset(r, ch * 8, half_bytes)) = val;
+        if (lane == 0) {
+          // the unit's window-query rows (padded to nq_pad with the next rows, whose scores
+          // the epilogue discards) by TMA into the swizzled B-operand tile
+          if (qcount >= 2) ok = mbar_wait(&qempty_bar[qs], ((qcount >> 1) - 1) & 1, p.status, abort_flag);
+          if (ok) {
+            uint8_t* qb = qbuf + qs * qbytes;
+            const uint32_t half_bytes = (uint32_t)p.nq_pad * 128;
+            mbar_arrive_expect_tx(&qfull_bar[qs], qbytes);
+#pragma unroll
+            for (int h = 0; h < D / 64; ++h) tma_load_2d(qb + h * half_bytes, &qmap, &qfull_bar[qs], 64 * h, unit * p.nq_rows);
+          }
         }
-        fence_proxy_async_smem();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&qfull_bar[qs]);
+        if (!__shfl_sync(0xffffffffu, ok, 0)) break;
         cur_unit = unit;
         ++qcount;
       }
@@ -144,8 +158,8 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
         const int qs = (qcount - 1) & 1;
         const int s = i % STAGES;
         if (!mbar_wait(&full_bar[s], (i / STAGES) & 1, p.status, abort_flag)) break;
-        const int acc = i & 1;
-        if (i >= 2 && !mbar_wait(&tempty_bar[acc], ((i >> 1) & 1) ^ 1, p.status, abort_flag)) break;
+        const int acc = i % n_acc;
+        if (i >= n_acc && !mbar_wait(&tempty_bar[acc], ((i / n_acc) & 1) ^ 1, p.status, abort_flag)) break;
         tc_fence_after();
         const uint32_t a_base = smem_u32(kstage + s * KTILE);
         const uint32_t b_base = smem_u32(qbuf + qs * qbytes);
@@ -167,46 +181,55 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       mbar_wait(drain_bar, 0, p.status, nullptr);
     }
   } else {
-    // ---------------------------------------------------------------- epilogue (warps 2..5)
+    // ---------------------------------------------------------------- epilogue (2 groups of 4 warps)
+    const int grp = (warp - 2) >> 2;            // group 0: warps 2-5, group 1: warps 6-9; tiles i % 2 == grp
     const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
-    const int ep_tid = tid - 64;
+    const int ep_tid = (warp - 2 - 4 * grp) * 32 + lane;
+    float* lse2_s = reinterpret_cast<float*>(smem + 1024 + grp * 2304);   // [288]
+    int* pw_s = reinterpret_cast<int*>(smem + 1024 + grp * 2304 + 1152);  // [288]
     const int win0 = p.t_ctx - p.window;        // position of window row 0
     int cur_unit = -1;
-    for (int i = 0; i < n; ++i) {
+    for (int i = grp; i < n; i += 2) {
       const int g = first + i;
       const int unit = g / p.tiles_per_unit, tt = g % p.tiles_per_unit;
       if (unit != cur_unit) {
-        named_bar(1, 128);
+        named_bar(1 + grp, 128);
         for (int c = ep_tid; c < 288; c += 128) {
           const bool real = c < p.nq_rows;
           lse2_s[c] = real ? __ldg(p.lse_win + (size_t)unit * p.nq_rows + c) * kLog2e : INFINITY;
           pw_s[c] = real ? win0 + c % p.window : -1;
         }
-        named_bar(1, 128);
+        named_bar(1 + grp, 128);
         cur_unit = unit;
       }
-      const int acc = i & 1;
-      if (!mbar_wait(&tfull_bar[acc], (i >> 1) & 1, p.status, abort_flag)) break;
+      const int acc = i % n_acc;
+      if (!mbar_wait(&tfull_bar[acc], (i / n_acc) & 1, p.status, abort_flag)) break;
       tc_fence_after();
       const int key_tile0 = p.n_sink + kSKeys * tt;
       const int key = key_tile0 + quad * 32 + lane;
       const bool causal = key_tile0 + kSKeys - 1 > win0;   // some key may follow a window row
       const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * p.acc_stride);
-      float sum = 0.f;
-      for (int c0 = 0; c0 < p.nq_pad; c0 += 32) {
-        float v[32];
-        tc_ld_32cols(taddr + c0, v);
+      float sum0 = 0.f, sum1 = 0.f, sum2 = 0.f, sum3 = 0.f;
+      for (int c0 = 0; c0 < p.nq_pad; c0 += 64) {
+        float v[64];
+        tc_ld_32cols(taddr + c0, *reinterpret_cast<float(*)[32]>(&v[0]));
+        tc_ld_32cols(taddr + c0 + 32, *reinterpret_cast<float(*)[32]>(&v[32]));
         tc_wait_ld();
-        const int ncol = min(32, p.nq_pad - c0);
-        if (ncol == 32 && !causal) {
+        const int ncol = min(64, p.nq_pad - c0);
+        if (ncol == 64 && !causal) {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) sum += fast_exp2(fmaf(v[j], p.scale_log2, -lse2_s[c0 + j]));
+          for (int j = 0; j < 64; j += 4) {
+            sum0 += fast_exp2(fmaf(v[j], p.scale_log2, -lse2_s[c0 + j]));
+            sum1 += fast_exp2(fmaf(v[j + 1], p.scale_log2, -lse2_s[c0 + j + 1]));
+            sum2 += fast_exp2(fmaf(v[j + 2], p.scale_log2, -lse2_s[c0 + j + 2]));
+            sum3 += fast_exp2(fmaf(v[j + 3], p.scale_log2, -lse2_s[c0 + j + 3]));
+          }
         } else {
 #pragma unroll
-          for (int j = 0; j < 32; ++j) {
+          for (int j = 0; j < 64; ++j) {
             if (j < ncol) {
               const float x = key <= pw_s[c0 + j] ? fmaf(v[j], p.scale_log2, -lse2_s[c0 + j]) : -INFINITY;
-              sum += fast_exp2(x);
+              sum0 += fast_exp2(x);
             }
           }
         }
@@ -214,7 +237,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty_bar[acc]);
-      if (key < p.mid_end) p.score[(size_t)unit * p.n_mid_pad + (key - p.n_sink)] = sum;
+      if (key < p.mid_end) p.score[(size_t)unit * p.n_mid_pad + (key - p.n_sink)] = (sum0 + sum1) + (sum2 + sum3);
     }
   }
 
@@ -232,39 +255,38 @@ struct TopkParams {
   int32_t* count_out;      // [units]
   int t_ctx, budget, n_sink, n_recent, chunk, n_mid_pad;
   int keep_all;            // budget >= t_ctx
+  int smem_items;          // item values staged in shared memory when n_items <= smem_items
 };
 
-__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* warp_sums, uint32_t* total) {
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  uint32_t x = v;
-#pragma unroll
-  for (int off = 1; off < 32; off <<= 1) {
-    const uint32_t y = __shfl_up_sync(0xffffffffu, x, off);
-    if (lane >= off) x += y;
-  }
-  if (lane == 31) warp_sums[warp] = x;
+// Exclusive scan of one value per warp (32 warps), result broadcast through smem.
+__device__ __forceinline__ uint32_t warp_totals_exclusive(uint32_t v, uint32_t* wsum, uint32_t* total) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) wsum[warp] = v;
   __syncthreads();
   if (warp == 0) {
-    uint32_t w = lane < (int)(blockDim.x >> 5) ? warp_sums[lane] : 0u;
+    const uint32_t w = wsum[lane];
     uint32_t incl = w;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const uint32_t y = __shfl_up_sync(0xffffffffu, incl, off);
       if (lane >= off) incl += y;
     }
-    warp_sums[lane] = incl - w;               // exclusive prefix of warp totals
+    wsum[lane] = incl - w;
     if (lane == 31) *total = incl;
   }
   __syncthreads();
-  const uint32_t r = warp_sums[warp] + x - v;
+  const uint32_t r = wsum[warp];
   __syncthreads();
   return r;
 }
 
-__global__ void __launch_bounds__(kTopkThreads) topk_kernel(const TopkParams p) {
+__global__ void __launch_bounds__(kTopkThreads, 1) topk_kernel(const TopkParams p) {
+  extern __shared__ uint32_t vals[];           // item values (fp32 bits) | candidates | samples
   __shared__ uint32_t hist[256];
-  __shared__ uint32_t warp_sums[32];
-  __shared__ uint32_t s_total, s_prefix, s_krem;
+  __shared__ uint32_t wsum[32];
+  __shared__ uint32_t s_total, s_prefix, s_krem, s_cnt;
+  grid_dependency_wait();
+  allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int unit = blockIdx.x;
   int32_t* out = p.idx_out + (size_t)unit * p.budget;
@@ -281,34 +303,166 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const TopkParams p) 
   const int n_items = (hi > lo) ? ((hi - 1) / s - c_first + 1) : 0;
   const int k = min(free / s, n_items);
   const float* sc = p.score + (size_t)unit * p.n_mid_pad;
+  const bool take_all = (k >= n_items), take_none = (k <= 0);
+  const bool ranked = !take_all && !take_none;
+  const bool staged = n_items <= p.smem_items;
 
-  auto item_value = [&](int i) -> uint32_t {
-    if (s == 1) return __float_as_uint(__ldcg(sc + i));
-    const int c = c_first + i;
-    const int a = max(c * s, lo), b = min(c * s + s, hi);
-    float v = 0.f;
-    for (int q = a; q < b; ++q) v += __ldcg(sc + (q - lo));
-    return __float_as_uint(v);
-  };
-  auto item_members = [&](int i, int& a, int& b) {
+  auto members = [&](int i, int& a, int& b) {
     const int c = c_first + i;
     a = max(c * s, lo);
     b = min(c * s + s, hi);
   };
+  auto value_global = [&](int i) -> uint32_t {
+    if (s == 1) return __float_as_uint(__ldcg(sc + i));
+    int a, b;
+    members(i, a, b);
+    float v = 0.f;
+    for (int q = a; q < b; ++q) v += __ldcg(sc + (q - lo));
+    return __float_as_uint(v);
+  };
+  if (ranked && staged) {
+    if (s == 1) {
+      const int n4 = n_items / 4;
+      const float4* sc4 = reinterpret_cast<const float4*>(sc);
+      for (int i = tid; i < n4; i += kTopkThreads) {
+        const float4 v = __ldcg(sc4 + i);
+        vals[4 * i] = __float_as_uint(v.x);
+        vals[4 * i + 1] = __float_as_uint(v.y);
+        vals[4 * i + 2] = __float_as_uint(v.z);
+        vals[4 * i + 3] = __float_as_uint(v.w);
+      }
+      for (int i = 4 * n4 + tid; i < n_items; i += kTopkThreads) vals[i] = __float_as_uint(__ldcg(sc + i));
+    } else {
+      for (int i = tid; i < n_items; i += kTopkThreads) vals[i] = value_global(i);
+    }
+    __syncthreads();
+  }
+  auto val = [&](int i) -> uint32_t { return staged ? vals[i] : value_global(i); };
 
-  // ---- radix select: value bits of the k-th largest item, and how many equal ones to take
-  uint32_t prefix = 0, mask = 0, krem = (uint32_t)k;
-  const bool take_all = (k >= n_items), take_none = (k <= 0);
-  if (!take_all && !take_none) {
+  // ---- value bits of the k-th largest item (tau) and how many items equal to tau to take (krem)
+  // Linear histogram between the block's min and max value: bins are monotone in the value,
+  // so the k-th largest lies in the bin where the count from the top reaches k; its items
+  // are few and are ranked exactly by (value desc, position asc).
+  uint32_t prefix = 0, krem = (uint32_t)k;
+  bool found = false, simple_eq = false;
+  if (ranked && staged) {
+    uint32_t* bins = reinterpret_cast<uint32_t*>(vals + ((p.smem_items + 1) & ~1));   // [kBins]
+    uint64_t* cand = reinterpret_cast<uint64_t*>(bins + kBins);                       // [kBinCandMax]
+    float lmin = INFINITY, lmax = -INFINITY;
+    for (int i = tid; i < n_items; i += kTopkThreads) {
+      const float v = __uint_as_float(vals[i]);
+      lmin = fminf(lmin, v);
+      lmax = fmaxf(lmax, v);
+    }
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, off));
+      lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, off));
+    }
+    __shared__ float s_min[32], s_max[32];
+    __shared__ uint32_t s_bin, s_above, s_nc, s_taukey, s_eq_take, s_eq_all;
+    if (lane == 0) {
+      s_min[warp] = lmin;
+      s_max[warp] = lmax;
+    }
+    for (int i = tid; i < kBins; i += kTopkThreads) bins[i] = 0;
+    if (tid == 0) {
+      s_nc = 0;
+      s_eq_take = 0;
+      s_eq_all = 0;
+      s_bin = 0xFFFFFFFFu;
+    }
+    __syncthreads();
+    float vmin = s_min[0], vmax = s_max[0];
+    for (int w = 1; w < 32; ++w) {
+      vmin = fminf(vmin, s_min[w]);
+      vmax = fmaxf(vmax, s_max[w]);
+    }
+    const float scale = vmax > vmin ? (float)(kBins - 1) / (vmax - vmin) : 0.f;
+    auto bin_of = [&](uint32_t u) -> int {
+      return min(kBins - 1, (int)((__uint_as_float(u) - vmin) * scale));
+    };
+    for (int i = tid; i < n_items; i += kTopkThreads) atomicAdd(&bins[bin_of(vals[i])], 1u);
+    __syncthreads();
+    // items in the bins of higher threads: total minus the inclusive prefix over threads
+    uint32_t mine = 0;
+#pragma unroll
+    for (int j = 0; j < kBins / kTopkThreads; ++j) mine += bins[tid * (kBins / kTopkThreads) + j];
+    uint32_t incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t z = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += z;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t w = wsum[lane];
+      uint32_t c = w;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+        if (lane >= off) c += z;
+      }
+      wsum[lane] = c - w;
+      if (lane == 31) s_total = c;
+    }
+    __syncthreads();
+    uint32_t above = s_total - (wsum[warp] + incl);   // items in bins above this thread's bins
+    for (int j = kBins / kTopkThreads - 1; j >= 0; --j) {
+      const int bidx = tid * (kBins / kTopkThreads) + j;
+      const uint32_t h = bins[bidx];
+      if (above < (uint32_t)k && (uint32_t)k <= above + h) {
+        s_bin = (uint32_t)bidx;
+        s_above = above;
+      }
+      above += h;
+    }
+    __syncthreads();
+    const int bstar = (int)s_bin;
+    const uint32_t nc = bins[bstar];
+    if (nc <= (uint32_t)kBinCandMax) {
+      for (int i = tid; i < n_items; i += kTopkThreads) {
+        const uint32_t u = vals[i];
+        if (bin_of(u) == bstar) cand[atomicAdd(&s_nc, 1u)] = (static_cast<uint64_t>(u) << 32) | (0xFFFFFFFFu - (uint32_t)i);
+      }
+      __syncthreads();
+      const uint32_t m = (uint32_t)k - s_above;       // rank (1-based) of the k-th item inside the bin
+      for (int i = tid; i < (int)nc; i += kTopkThreads) {
+        const uint64_t key = cand[i];
+        uint32_t rank = 0;
+        for (int j = 0; j < (int)nc; ++j) rank += cand[j] > key;
+        if (rank == m - 1) s_taukey = static_cast<uint32_t>(key >> 32);
+      }
+      __syncthreads();
+      prefix = s_taukey;
+      for (int i = tid; i < (int)nc; i += kTopkThreads) {
+        const uint64_t key = cand[i];
+        if (static_cast<uint32_t>(key >> 32) != prefix) continue;
+        uint32_t rank = 0;
+        for (int j = 0; j < (int)nc; ++j) rank += cand[j] > key;
+        atomicAdd(&s_eq_all, 1u);
+        if (rank < m) atomicAdd(&s_eq_take, 1u);
+      }
+      __syncthreads();
+      krem = s_eq_take;
+      simple_eq = (s_eq_take == s_eq_all);
+      found = true;
+    }
+  }
+  // ---- otherwise radix select (MSB first, 8 bits per pass)
+  uint32_t mask = 0;
+  const int n_round = (n_items + kTopkThreads - 1) / kTopkThreads * kTopkThreads;
+  if (ranked && !found) {
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
-      for (int i = tid; i < 256; i += kTopkThreads) hist[i] = 0;
+      if (tid < 256) hist[tid] = 0;
       __syncthreads();
-      for (int base = 0; base < n_items; base += kTopkThreads) {
-        const int i = base + tid;
+#pragma unroll 4
+      for (int i = tid; i < n_round; i += kTopkThreads) {
         uint32_t digit = 256;
         if (i < n_items) {
-          const uint32_t u = item_value(i);
+          const uint32_t u = val(i);
           if ((u & mask) == prefix) digit = (u >> shift) & 255u;
         }
         const uint32_t peers = __match_any_sync(0xffffffffu, digit);
@@ -316,11 +470,10 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const TopkParams p) 
       }
       __syncthreads();
       if (warp == 0) {
-        // lane l owns digits 8l .. 8l+7; count of items with a larger digit than lane l's range
         uint32_t local = 0;
 #pragma unroll
         for (int j = 0; j < 8; ++j) local += hist[8 * lane + j];
-        uint32_t suffix = local;   // inclusive suffix sum over lanes >= lane
+        uint32_t suffix = local;   // items whose digit is >= 8*lane
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
           const uint32_t y = __shfl_down_sync(0xffffffffu, suffix, off);
@@ -343,48 +496,82 @@ __global__ void __launch_bounds__(kTopkThreads) topk_kernel(const TopkParams p) 
       prefix = s_prefix;
       krem = s_krem;
       mask |= 0xFFu << shift;
-      __syncthreads();
     }
   }
-  const uint32_t tau = prefix;
+  const uint32_t tau = prefix;   // value bits of the k-th largest item; take krem of the equal ones
 
-  // ---- compaction in item order (contiguous ranges per thread keep the output ascending)
-  const int per = (n_items + kTopkThreads - 1) / kTopkThreads;
-  const int i0 = min(n_items, tid * per), i1 = min(n_items, i0 + per);
-  uint32_t eq_local = 0;
-  if (!take_all && !take_none)
-    for (int i = i0; i < i1; ++i) eq_local += (item_value(i) == tau);
-  const uint32_t eq_base = block_exclusive_scan(eq_local, warp_sums, &s_total);
-  auto selected = [&](int i, uint32_t& eq_seen) -> bool {
-    if (take_all) return true;
-    if (take_none) return false;
-    const uint32_t u = item_value(i);
-    if (u > tau) return true;
-    if (u == tau) return (eq_base + eq_seen++) < krem;
-    return false;
+  // ---- compaction in item order: warp w owns items [w*ipw, (w+1)*ipw), lane-interleaved rows
+  const int ipw = (n_items + 32 * 32 - 1) / (32 * 32) * 32;
+  const int w0 = warp * ipw, w1 = min(n_items, w0 + ipw);
+  const uint32_t lt_mask = (1u << lane) - 1u;
+  uint32_t eq_count = 0;
+  const bool need_eq = ranked && !simple_eq;      // some items equal to tau are left out
+  if (need_eq)
+    for (int j = w0; j < w1; j += 32) {
+      const int i = j + lane;
+      const bool eq = i < w1 && val(i) == tau;
+      eq_count += __popc(__ballot_sync(0xffffffffu, eq));
+    }
+  const uint32_t eq_base = warp_totals_exclusive(eq_count, wsum, &s_total);
+  auto select_row = [&](int j, uint32_t& eq_run, int& npos) -> bool {
+    const int i = j + lane;
+    bool sel = false;
+    bool eq = false;
+    if (i < w1) {
+      if (take_all) {
+        sel = true;
+      } else if (ranked) {
+        const uint32_t u = val(i);
+        eq = (u == tau);
+        sel = u > tau;
+      }
+    }
+    const uint32_t bal = __ballot_sync(0xffffffffu, eq);
+    if (eq) sel = need_eq ? (eq_run + __popc(bal & lt_mask)) < krem : true;
+    eq_run += __popc(bal);
+    npos = 0;
+    if (sel) {
+      int a, b;
+      members(i, a, b);
+      npos = b - a;
+    }
+    return sel;
   };
-  uint32_t npos_local = 0;
+  uint32_t pos_count = 0;
   {
-    uint32_t eq_seen = 0;
-    for (int i = i0; i < i1; ++i)
-      if (selected(i, eq_seen)) {
-        int a, b;
-        item_members(i, a, b);
-        npos_local += (uint32_t)(b - a);
-      }
+    uint32_t eq_run = eq_base;
+    for (int j = w0; j < w1; j += 32) {
+      int npos;
+      select_row(j, eq_run, npos);
+      int sum = npos;
+#pragma unroll
+      for (int off = 16; off > 0; off >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, off);
+      pos_count += (uint32_t)sum;
+    }
   }
-  const uint32_t pos_base = block_exclusive_scan(npos_local, warp_sums, &s_total);
-  const uint32_t n_chosen = s_total;
+  const uint32_t pos_base = warp_totals_exclusive(pos_count, wsum, &s_total);
+  const int n_chosen = (int)s_total;
   {
-    uint32_t eq_seen = 0, w = (uint32_t)lo + pos_base;
-    for (int i = i0; i < i1; ++i)
-      if (selected(i, eq_seen)) {
-        int a, b;
-        item_members(i, a, b);
-        for (int q = a; q < b; ++q) out[w++] = q;
+    uint32_t eq_run = eq_base, w = (uint32_t)lo + pos_base;
+    for (int j = w0; j < w1; j += 32) {
+      int npos;
+      const bool sel = select_row(j, eq_run, npos);
+      int incl = npos;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off) incl += y;
       }
+      if (sel) {
+        int a, b;
+        members(j + lane, a, b);
+        int o = (int)w + incl - npos;
+        for (int q = a; q < b; ++q) out[o++] = q;
+      }
+      w += (uint32_t)__shfl_sync(0xffffffffu, incl, 31);
+    }
   }
-  const int count = lo + (int)n_chosen + p.n_recent;
+  const int count = lo + n_chosen + p.n_recent;
   for (int i = tid; i < lo; i += kTopkThreads) out[i] = i;
   for (int i = tid; i < p.n_recent; i += kTopkThreads) out[lo + n_chosen + i] = hi + i;
   for (int i = count + tid; i < p.budget; i += kTopkThreads) out[i] = -1;
@@ -426,8 +613,10 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   plan->tiles_per_cta = (plan->total_tiles + plan->grid - 1) / plan->grid;
   plan->grid = std::max(1, (plan->total_tiles + plan->tiles_per_cta - 1) / plan->tiles_per_cta);
   plan->stages = kSStages;
-  plan->tmem_cols = pow2_at_least(2u * (uint32_t)align_up(plan->nq_pad, 32));
-  plan->smem_bytes = 1024 + 4096 + 2 * (size_t)plan->nq_pad * s.head_dim * 2 +
+  const uint32_t acc_stride = (uint32_t)align_up(plan->nq_pad, 32);
+  plan->n_acc = 4u * acc_stride <= 512u ? 4 : 2;
+  plan->tmem_cols = pow2_at_least((uint32_t)plan->n_acc * acc_stride);
+  plan->smem_bytes = 1024 + kSQOffset + 2 * (size_t)plan->nq_pad * s.head_dim * 2 +
                      (size_t)kSStages * kSKeys * s.head_dim * 2;
   plan->score_bytes = plan->need_scores ? align_up((size_t)units * plan->n_mid_pad * 4, 256) : 0;
   plan->lse_bytes = align_up((size_t)s.batch * s.h_q * window * 4, 256);
@@ -461,8 +650,10 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
       if (err != cudaSuccess) return err;
       lse = lse_buf;
     }
-    CUtensorMap kmap;
+    CUtensorMap kmap, qmap;
     err = make_cache_map(&kmap, k_cache, units, s.t_cap, s.t_ctx, s.head_dim, kSKeys);
+    if (err != cudaSuccess) return err;
+    err = make_rows_map(&qmap, q_window, (long long)units * plan.nq_rows, s.head_dim, plan.nq_pad);
     if (err != cudaSuccess) return err;
     ScoreParams p;
     p.q_win = static_cast<const __nv_bfloat16*>(q_window);
@@ -480,13 +671,14 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
     p.total_tiles = plan.total_tiles;
     p.tiles_per_cta = plan.tiles_per_cta;
     p.acc_stride = (int)align_up(plan.nq_pad, 32);
+    p.n_acc = plan.n_acc;
     p.tmem_cols = plan.tmem_cols;
     p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
     void* fn = score_fn(s.head_dim);
     err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
     if (err != cudaSuccess) return err;
-    void* args[] = {&p, &kmap};
-    err = cudaLaunchKernel(fn, dim3(plan.grid), dim3(kSThreads), args, plan.smem_bytes, stream);
+    void* args[] = {&p, &kmap, &qmap};
+    err = launch_kernel(fn, dim3(plan.grid), dim3(kSThreads), plan.smem_bytes, stream, args, 0);
     if (err != cudaSuccess) return err;
   }
   TopkParams tp;
@@ -500,8 +692,17 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
   tp.chunk = chunk;
   tp.n_mid_pad = plan.n_mid_pad;
   tp.keep_all = plan.keep_all ? 1 : 0;
-  topk_kernel<<<units, kTopkThreads, 0, stream>>>(tp);
-  return cudaGetLastError();
+  const int extra = kBins * 4 + kBinCandMax * 8 + 16;      // histogram + boundary-bin candidates
+  const int max_items = (kTopkSmemBytes - extra) / 4;
+  const int n_items = plan.n_mid;                     // upper bound for chunk mode as well
+  tp.smem_items = std::min(n_items, max_items);
+  const size_t smem = (size_t)((tp.smem_items + 1) & ~1) * 4 + extra;
+  err = cudaFuncSetAttribute(reinterpret_cast<void*>(&topk_kernel), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)smem);
+  if (err != cudaSuccess) return err;
+  void* targs[] = {&tp};
+  return launch_kernel(reinterpret_cast<void*>(&topk_kernel), dim3(units), dim3(kTopkThreads), smem, stream, targs,
+                       0);
 }
 
 }  // namespace bd
