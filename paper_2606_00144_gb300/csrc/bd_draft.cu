@@ -10,9 +10,10 @@
 //      (unused rows zero-filled) and the four warps run the mma.sync sub-tile code shared
 //      with the verify kernel (bd_attn_warp.cuh), the G heads of the GQA group forming one
 //      n8 query tile;
-//   3. the CTAs' normalised partials are merged through distributed shared memory by the
-//      cluster's rank-0 CTA (log-sum-exp), which writes the bf16 output: no global
-//      partials, fences or atomics.
+//   3. every CTA stores its normalised partial straight into the shared memory of the
+//      cluster's rank-0 CTA (distributed shared memory); after one cluster barrier rank 0
+//      merges them (log-sum-exp) from its own shared memory and writes the bf16 output:
+//      no global partials, fences or atomics.
 // Launched with programmatic dependent launch: the grid-dependency wait is the first thing
 // a CTA does, and the next kernel may be scheduled as soon as every CTA has passed it.
 #include <cooperative_groups.h>
@@ -28,10 +29,10 @@ namespace cg = cooperative_groups;
 
 namespace bd {
 
-constexpr int kDRows = 80;        // rows per shared-memory tile (5 sub-tiles of 16)
-constexpr int kDSubs = kDRows / 16;
-constexpr int kDThreads = 128;    // 4 warps
-constexpr int kDMaxCluster = 8;   // portable cluster size
+constexpr int kDRows = 80;        // rows per shared-memory tile: 5 sub-tiles of 16, one per warp
+constexpr int kDWarps = kDRows / 16;
+constexpr int kDThreads = 32 * kDWarps;
+constexpr int kDMaxCluster = 8;   // CTAs per (sequence, KV head): the portable cluster size
 
 struct DraftParams {
   const __nv_bfloat16* q;      // [units * G][D]
@@ -51,11 +52,12 @@ template <int D, int G>
 struct DraftSmem {
   static constexpr uint32_t TILE_BYTES = kDRows * D * 2;
   static constexpr uint32_t STAGE_BYTES = 2 * TILE_BYTES;                 // K and V
-  static constexpr size_t kMerge = (size_t)(3 * 4 * 8) * 4 + (size_t)4 * 8 * (D + 4) * 4;
-  // stages (the warp-merge scratch reuses them) | rowpos [2][kDRows] | partial o [G][D], lse [G]
-  static size_t bytes(int n_stage) {
+  static constexpr size_t kMerge = (size_t)(3 * kDWarps * 8) * 4 + (size_t)kDWarps * 8 * (D + 4) * 4;
+  // stages (the warp-merge scratch reuses them) | rowpos [2][kDRows] |
+  // partials of the cluster's CTAs [C][G*D + G] (used in rank 0 only)
+  static size_t bytes(int n_stage, int cluster) {
     const size_t stages = std::max<size_t>((size_t)n_stage * STAGE_BYTES, kMerge);
-    return 1024 + stages + 2 * kDRows * 4 + (size_t)G * D * 4 + G * 4 + 16;
+    return 1024 + stages + 2 * kDRows * 4 + (size_t)cluster * (G * D + G) * 4 + 16;
   }
 };
 
@@ -74,16 +76,17 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
                                                                                : kMergeBytes;
   uint8_t* stage = smem;                                                  // n_stage x (K, V)
   int* rowpos = reinterpret_cast<int*>(smem + stage_bytes);               // [2][kDRows]
-  float* part_o = reinterpret_cast<float*>(rowpos + 2 * kDRows);          // [G][D]
-  float* part_lse = part_o + G * D;                                       // [G]
+  float* parts = reinterpret_cast<float*>(rowpos + 2 * kDRows);           // [C][G*D + G]
   float* m_s = reinterpret_cast<float*>(stage);                           // warp-merge scratch
-  float* l_s = m_s + 4 * 8;
-  float* f_s = l_s + 4 * 8;
-  float* o_s = f_s + 4 * 8;
+  float* l_s = m_s + kDWarps * 8;
+  float* f_s = l_s + kDWarps * 8;
+  float* o_s = f_s + kDWarps * 8;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int split = blockIdx.x, unit = blockIdx.y;
   const int32_t* iunit = p.idx + (size_t)unit * p.budget;
+  // announce this CTA has started; the matching wait precedes the first remote store
+  if (p.n_split > 1) asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
   const int e_begin = split * p.rows_per_split;
   // count and the first tile's indices in flight together
   int idx_pref = -1;
@@ -160,8 +163,8 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     const int nrows = min(kDRows, e_end - (e_begin + t * kDRows));
     const uint32_t kbase = smem_u32(stage + b * L::STAGE_BYTES);
     const int* rp = rowpos + b * kDRows;
-    for (int sub = warp; sub < kDSubs && 16 * sub < nrows; sub += 4) {
-      const int kb = 16 * sub;
+    if (16 * warp < nrows) {
+      const int kb = 16 * warp;
       wa.step(kbase, kbase + L::TILE_BYTES, HALF_BYTES, kb, bq, p.scale_log2, lane, [&](int ko, int, int) {
         const int r = kb + ko;
         return r < nrows && rp[r] >= 0;
@@ -179,46 +182,46 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   __syncthreads();
   const size_t row0 = (size_t)unit * G;
   if (p.n_split == 1) {
-    merge_warps_and_store<D, 4, true>(m_s, l_s, f_s, o_s, 8, G, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D, true,
-                                      tid, kDThreads, 0);
+    merge_warps_and_store<D, kDWarps, true>(m_s, l_s, f_s, o_s, 8, G, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D,
+                                            true, tid, kDThreads, 0);
     return;
   }
-  merge_warps_and_store<D, 4, true>(m_s, l_s, f_s, o_s, 8, G, part_lse, part_o, false, tid, kDThreads, 0);
-
   // ---------------------------------------------------------------- cluster merge (DSMEM)
   cg::cluster_group cluster = cg::this_cluster();
-  cluster.sync();                                  // every CTA's partial is in its shared memory
-  if (cluster.block_rank() == 0) {
-    const int C = p.n_split;
-    float* wts = o_s;                              // [C][G] weights, then scale
-    if (tid < G) {
-      float mx = -INFINITY;
-      for (int r = 0; r < C; ++r) mx = fmaxf(mx, *cluster.map_shared_rank(part_lse + tid, r));
-      float tot = 0.f;
-      for (int r = 0; r < C; ++r) {
-        const float l = *cluster.map_shared_rank(part_lse + tid, r);
-        const float w = mx == -INFINITY ? 0.f : fast_exp2((l - mx) * kLog2e);
-        wts[r * G + tid] = w;
-        tot += w;
-      }
-      const float inv = tot > 0.f ? 1.f / tot : 0.f;
-      for (int r = 0; r < C; ++r) wts[r * G + tid] *= inv;
-      if (p.lse) p.lse[row0 + tid] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
+  const int C = p.n_split;
+  const int rank = (int)cluster.block_rank();
+  float* slot = cluster.map_shared_rank(parts, 0) + (size_t)rank * (G * D + G);   // in rank 0
+  asm volatile("barrier.cluster.wait.aligned;" ::: "memory");          // every CTA is running
+  merge_warps_and_store<D, kDWarps, true>(m_s, l_s, f_s, o_s, 8, G, slot + G * D, slot, false, tid, kDThreads, 0);
+  cluster.sync();                                  // all partials have landed in rank 0
+  if (rank != 0) return;
+  float* wts = o_s;                                // [C][G] merge weights
+  if (tid < G) {
+    float mx = -INFINITY;
+    for (int r = 0; r < C; ++r) mx = fmaxf(mx, parts[r * (G * D + G) + G * D + tid]);
+    float tot = 0.f;
+    for (int r = 0; r < C; ++r) {
+      const float l = parts[r * (G * D + G) + G * D + tid];
+      const float w = mx == -INFINITY ? 0.f : fast_exp2((l - mx) * kLog2e);
+      wts[r * G + tid] = w;
+      tot += w;
     }
-    __syncthreads();
-    for (int i = tid; i < G * (D / 2); i += kDThreads) {
-      const int g = i / (D / 2), d = (i % (D / 2)) * 2;
-      float a0 = 0.f, a1 = 0.f;
-      for (int r = 0; r < C; ++r) {
-        const float w = wts[r * G + g];
-        const float2 v = *reinterpret_cast<const float2*>(cluster.map_shared_rank(part_o + g * D + d, r));
-        a0 += w * v.x;
-        a1 += w * v.y;
-      }
-      *reinterpret_cast<uint32_t*>(p.o + (row0 + g) * D + d) = pack_bf16x2(a0, a1);
-    }
+    const float inv = tot > 0.f ? 1.f / tot : 0.f;
+    for (int r = 0; r < C; ++r) wts[r * G + tid] *= inv;
+    if (p.lse) p.lse[row0 + tid] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
   }
-  cluster.sync();                                  // partials stay alive until rank 0 has read them
+  __syncthreads();
+  for (int i = tid; i < G * (D / 2); i += kDThreads) {
+    const int g = i / (D / 2), d = (i % (D / 2)) * 2;
+    float a0 = 0.f, a1 = 0.f;
+    for (int r = 0; r < C; ++r) {
+      const float w = wts[r * G + g];
+      const float2 v = *reinterpret_cast<const float2*>(parts + r * (G * D + G) + g * D + d);
+      a0 += w * v.x;
+      a1 += w * v.y;
+    }
+    *reinterpret_cast<uint32_t*>(p.o + (row0 + g) * D + d) = pack_bf16x2(a0, a1);
+  }
 }
 
 // ============================================================================ host side
@@ -233,9 +236,9 @@ DraftFn pick(int d, int g) {
 #undef BD_DK
   return nullptr;
 }
-size_t smem_bytes(int d, int g, int n_stage) {
+size_t smem_bytes(int d, int g, int n_stage, int cluster) {
 #define BD_DS(DD, GG) \
-  if (d == DD && g == GG) return DraftSmem<DD, GG>::bytes(n_stage);
+  if (d == DD && g == GG) return DraftSmem<DD, GG>::bytes(n_stage, cluster);
   BD_DS(64, 1) BD_DS(64, 2) BD_DS(64, 4) BD_DS(64, 8)
   BD_DS(128, 1) BD_DS(128, 2) BD_DS(128, 4) BD_DS(128, 8)
 #undef BD_DS
@@ -283,9 +286,10 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const int g = s.h_q / s.h_kv;
   void* fn = pick(s.head_dim, g);
-  const size_t smem = smem_bytes(s.head_dim, g, p.n_stage);
+  const size_t smem = smem_bytes(s.head_dim, g, p.n_stage, plan.n_split);
   cudaError_t err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
+
   void* args[] = {&p};
   return launch_kernel(fn, dim3(plan.n_split, units), dim3(kDThreads), smem, stream, args,
                        plan.n_split > 1 ? plan.n_split : 0);
