@@ -309,19 +309,23 @@ def gpu_arm(args):
     step.run()
     torch.cuda.synchronize()
     S = graph_len(args.steps, args.graph_steps)
+    g_main = capture(lambda i: step.run(), S)
     marks = [[timing_event() for _ in range(4)] for _ in range(S)]
-    g_main = capture(lambda i: step.run(marks[i]), S)
+    g_marked = capture(lambda i: step.run(marks[i]), S)
     g_warm = capture(lambda i: step.run(), 1)
     for _ in range(args.warmup):
         g_warm.replay()
     torch.cuda.synchronize()
 
+    # timed region: K steps, kernels only (programmatic dependent launch between them)
     sampler = ClockSampler(local)
     sampler.start()
     ms = timed_replays([g_main] * (args.steps // S), world)
     clocks = sampler.stop()
     ms = max_over_ranks(ms, world)
-    # per-phase durations: the S steps of the last replay inside the timed region
+    # per-phase durations: the same K steps with event nodes between the phases (which
+    # also stop the dependent-launch overlap at those boundaries); the last replay's marks
+    timed_replays([g_marked] * (args.steps // S), world)
     ph = {"select": [], "draft": [], "verify": []}
     for i in range(S):
         e = [m[0] for m in marks[i]]
