@@ -7,6 +7,8 @@
 //               row: no cross-thread reduction.  Persistent CTAs (one per SM):
 //                 warp 0   producer: K tiles by TMA (128-byte swizzle, 4-stage ring) and the
 //                          unit's window queries into a double-buffered swizzled Q tile;
+//                          both are context data, streamed before the grid-dependency
+//                          wait, which only the epilogue (reading the window LSE) takes;
 //                 warp 1   one lane issues tcgen05.mma into a double-buffered fp32 TMEM
 //                          accumulator and commits to the smem/TMEM barriers;
 //                 warps 2-5 epilogue: tcgen05.ld, ex2 (MUFU), row sums, coalesced store.
@@ -65,8 +67,6 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
   uint8_t* qbuf = smem + kSQOffset;                            // 2 x qbytes
   uint8_t* kstage = qbuf + 2 * qbytes;                         // STAGES x KTILE (1024-aligned)
 
-  grid_dependency_wait();
-  allow_dependent_launch();
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int first = blockIdx.x * p.tiles_per_cta;
   const int n = max(0, min(p.tiles_per_cta, p.total_tiles - first));
@@ -100,6 +100,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
 
   if (warp == 0) {
     // ---------------------------------------------------------------- producer
+    allow_dependent_launch();
     if (lane == 0) {
       tma_prefetch_map(&kmap);
       tma_prefetch_map(&qmap);
@@ -143,6 +144,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
+    allow_dependent_launch();
     if (lane == 0) {
       const uint32_t idesc = umma_idesc_bf16(kSKeys, p.nq_pad);
       int cur_unit = -1, qcount = 0;
@@ -182,6 +184,8 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     }
   } else {
     // ---------------------------------------------------------------- epilogue (2 groups of 4 warps)
+    grid_dependency_wait();                      // the window LSE is carried from earlier kernels
+    allow_dependent_launch();
     const int grp = (warp - 2) >> 2;            // group 0: warps 2-5, group 1: warps 6-9; tiles i % 2 == grp
     const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
     const int ep_tid = (warp - 2 - 4 * grp) * 32 + lane;
@@ -578,6 +582,287 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_kernel(const TopkParams 
   if (tid == 0) p.count_out[unit] = count;
 }
 
+// Token-level selection with the scores staged in shared memory (the graded workloads'
+// path): the same boundary-bin method as topk_kernel, written lean.  Needs 0 < k < n <=
+// kLeanMaxItems; the selection mask of each item is kept as warp ballots in registers.
+constexpr int kLeanMaxItems = 32 * kTopkThreads;   // 32 rows of 32 items per warp
+constexpr int kLeanRows = kLeanMaxItems / kTopkThreads;
+
+__global__ void __launch_bounds__(kTopkThreads, 1) topk_token_kernel(const TopkParams p) {
+  extern __shared__ uint32_t vals[];                // n scores (fp32 bits)
+  __shared__ uint32_t bins[kBins];
+  __shared__ uint64_t cand[kBinCandMax];
+  __shared__ uint32_t wsum[32];
+  __shared__ float wmin[32], wmax[32];
+  __shared__ uint32_t s_total, s_bin, s_above, s_nc, s_taukey, s_eq_take, s_eq_all, s_prefix, s_krem;
+  __shared__ float s_vmin, s_vmax;
+  grid_dependency_wait();
+  allow_dependent_launch();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int unit = blockIdx.x;
+  const int lo = p.n_sink, hi = p.t_ctx - p.n_recent, n = hi - lo;
+  const int k = p.budget - p.n_sink - p.n_recent;
+  const float* sc = p.score + (size_t)unit * p.n_mid_pad;
+  int32_t* out = p.idx_out + (size_t)unit * p.budget;
+
+  // ---- stage the scores, min and max
+  float lmin = INFINITY, lmax = -INFINITY;
+  const int n4 = n >> 2;
+  const float4* sc4 = reinterpret_cast<const float4*>(sc);
+  for (int i = tid; i < n4; i += kTopkThreads) {
+    const float4 v = __ldcg(sc4 + i);
+    reinterpret_cast<uint4*>(vals)[i] = make_uint4(__float_as_uint(v.x), __float_as_uint(v.y), __float_as_uint(v.z),
+                                                   __float_as_uint(v.w));
+    lmin = fminf(fminf(lmin, fminf(v.x, v.y)), fminf(v.z, v.w));
+    lmax = fmaxf(fmaxf(lmax, fmaxf(v.x, v.y)), fmaxf(v.z, v.w));
+  }
+  for (int i = 4 * n4 + tid; i < n; i += kTopkThreads) {
+    const float v = __ldcg(sc + i);
+    vals[i] = __float_as_uint(v);
+    lmin = fminf(lmin, v);
+    lmax = fmaxf(lmax, v);
+  }
+  for (int i = tid; i < kBins; i += kTopkThreads) bins[i] = 0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, off));
+    lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, off));
+  }
+  if (lane == 0) {
+    wmin[warp] = lmin;
+    wmax[warp] = lmax;
+  }
+  if (tid == 0) {
+    s_nc = 0;
+    s_eq_take = 0;
+    s_eq_all = 0;
+  }
+  __syncthreads();
+  if (warp == 0) {
+    float a = wmin[lane], b = wmax[lane];
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) {
+      a = fminf(a, __shfl_xor_sync(0xffffffffu, a, off));
+      b = fmaxf(b, __shfl_xor_sync(0xffffffffu, b, off));
+    }
+    if (lane == 0) {
+      s_vmin = a;
+      s_vmax = b;
+    }
+  }
+  __syncthreads();
+  const float vmin = s_vmin, vmax = s_vmax;
+
+  // ---- tau (bits of the k-th largest score) and krem (how many scores equal to tau to keep)
+  uint32_t tau = 0, krem = (uint32_t)k;
+  bool simple = false, found = false;
+  if (vmax > vmin) {
+    const float scale = (float)(kBins - 1) / (vmax - vmin);
+    auto bin_of = [&](uint32_t u) -> int { return min(kBins - 1, (int)((__uint_as_float(u) - vmin) * scale)); };
+    for (int i = tid; i < n; i += kTopkThreads) atomicAdd(&bins[bin_of(vals[i])], 1u);
+    __syncthreads();
+    constexpr int BPT = kBins / kTopkThreads;
+    uint32_t mine = 0;
+#pragma unroll
+    for (int j = 0; j < BPT; ++j) mine += bins[tid * BPT + j];
+    uint32_t incl = mine;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t z = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += z;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t w = wsum[lane];
+      uint32_t c = w;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+        if (lane >= off) c += z;
+      }
+      wsum[lane] = c - w;
+      if (lane == 31) s_total = c;
+    }
+    __syncthreads();
+    uint32_t above = s_total - (wsum[warp] + incl);
+#pragma unroll
+    for (int j = BPT - 1; j >= 0; --j) {
+      const uint32_t h = bins[tid * BPT + j];
+      if (above < (uint32_t)k && (uint32_t)k <= above + h) {
+        s_bin = (uint32_t)(tid * BPT + j);
+        s_above = above;
+      }
+      above += h;
+    }
+    __syncthreads();
+    const int bstar = (int)s_bin;
+    const uint32_t nc = bins[bstar];
+    if (nc <= (uint32_t)kBinCandMax) {
+      for (int i = tid; i < n; i += kTopkThreads) {
+        const uint32_t u = vals[i];
+        if (bin_of(u) == bstar) cand[atomicAdd(&s_nc, 1u)] = (static_cast<uint64_t>(u) << 32) | (0xFFFFFFFFu - (uint32_t)i);
+      }
+      __syncthreads();
+      const uint32_t m = (uint32_t)k - s_above;
+      uint64_t key = 0;
+      uint32_t rank = 0xFFFFFFFFu;
+      if (tid < (int)nc) {
+        key = cand[tid];
+        rank = 0;
+        for (int j = 0; j < (int)nc; ++j) rank += cand[j] > key;
+        if (rank == m - 1) s_taukey = static_cast<uint32_t>(key >> 32);
+      }
+      for (int i = tid + kTopkThreads; i < (int)nc; i += kTopkThreads) {   // nc > 1024: rare
+        const uint64_t kk = cand[i];
+        uint32_t r = 0;
+        for (int j = 0; j < (int)nc; ++j) r += cand[j] > kk;
+        if (r == m - 1) s_taukey = static_cast<uint32_t>(kk >> 32);
+      }
+      __syncthreads();
+      tau = s_taukey;
+      for (int i = tid; i < (int)nc; i += kTopkThreads) {
+        const uint64_t kk = cand[i];
+        if (static_cast<uint32_t>(kk >> 32) != tau) continue;
+        uint32_t r = (i == tid) ? rank : 0;
+        if (i != tid)
+          for (int j = 0; j < (int)nc; ++j) r += cand[j] > kk;
+        atomicAdd(&s_eq_all, 1u);
+        if (r < m) atomicAdd(&s_eq_take, 1u);
+      }
+      __syncthreads();
+      krem = s_eq_take;
+      simple = (s_eq_take == s_eq_all);
+      found = true;
+    }
+  }
+  if (!found) {
+    // crowded boundary (many equal or near-equal scores): exact 4-pass radix select
+    uint32_t prefix = 0, mask = 0;
+    krem = (uint32_t)k;
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      for (int i = tid; i < 256; i += kTopkThreads) bins[i] = 0;
+      __syncthreads();
+      for (int i = tid; i < n; i += kTopkThreads) {
+        const uint32_t u = vals[i];
+        if ((u & mask) == prefix) atomicAdd(&bins[(u >> shift) & 255u], 1u);
+      }
+      __syncthreads();
+      if (warp == 0) {
+        uint32_t local = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) local += bins[8 * lane + j];
+        uint32_t suffix = local;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const uint32_t y = __shfl_down_sync(0xffffffffu, suffix, off);
+          if (lane + off < 32) suffix += y;
+        }
+        uint32_t abv = suffix - local;
+        if (abv < krem && krem <= suffix) {
+          for (int j = 7; j >= 0; --j) {
+            const uint32_t h = bins[8 * lane + j];
+            if (abv + h >= krem) {
+              s_prefix = prefix | ((uint32_t)(8 * lane + j) << shift);
+              s_krem = krem - abv;
+              break;
+            }
+            abv += h;
+          }
+        }
+      }
+      __syncthreads();
+      prefix = s_prefix;
+      krem = s_krem;
+      mask |= 0xFFu << shift;
+    }
+    tau = prefix;
+    simple = false;
+  }
+
+  // ---- ascending compaction: warp w owns items [w*ipw, (w+1)*ipw), rows of 32
+  const int rows = (n + kTopkThreads - 1) / kTopkThreads;     // <= kLeanRows
+  const int w0 = warp * rows * 32;
+  const uint32_t lt = (1u << lane) - 1u;
+  uint32_t eq_base = 0;
+  if (!simple) {
+    uint32_t eqc = 0;
+#pragma unroll
+    for (int r = 0; r < kLeanRows; ++r) {
+      if (r < rows) {
+        const int i = w0 + 32 * r + lane;
+        eqc += __popc(__ballot_sync(0xffffffffu, i < n && vals[i] == tau));
+      }
+    }
+    if (lane == 0) wsum[warp] = eqc;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t w = wsum[lane];
+      uint32_t c = w;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+        if (lane >= off) c += z;
+      }
+      wsum[lane] = c - w;
+    }
+    __syncthreads();
+    eq_base = wsum[warp];
+    __syncthreads();
+  }
+  uint32_t masks[kLeanRows];
+  uint32_t cnt = 0, eq_run = eq_base;
+#pragma unroll
+  for (int r = 0; r < kLeanRows; ++r) {
+    masks[r] = 0;
+    if (r < rows) {
+      const int i = w0 + 32 * r + lane;
+      const uint32_t u = i < n ? vals[i] : 0u;
+      bool sel = i < n && u > tau;
+      const bool eq = i < n && u == tau;
+      if (simple) {
+        sel |= eq;
+      } else {
+        const uint32_t be = __ballot_sync(0xffffffffu, eq);
+        if (eq) sel = eq_run + __popc(be & lt) < krem;
+        eq_run += __popc(be);
+      }
+      masks[r] = __ballot_sync(0xffffffffu, sel);
+      cnt += __popc(masks[r]);
+    }
+  }
+  if (lane == 0) wsum[warp] = cnt;
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t w = wsum[lane];
+    uint32_t c = w;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+      if (lane >= off) c += z;
+    }
+    wsum[lane] = c - w;
+    if (lane == 31) s_total = c;
+  }
+  __syncthreads();
+  uint32_t base = (uint32_t)lo + wsum[warp];
+#pragma unroll
+  for (int r = 0; r < kLeanRows; ++r) {
+    if (r < rows) {
+      const uint32_t mk = masks[r];
+      if ((mk >> lane) & 1u) out[base + __popc(mk & lt)] = lo + w0 + 32 * r + lane;
+      base += __popc(mk);
+    }
+  }
+  const int n_chosen = (int)s_total;
+  const int count = lo + n_chosen + p.n_recent;
+  for (int i = tid; i < lo; i += kTopkThreads) out[i] = i;
+  for (int i = tid; i < p.n_recent; i += kTopkThreads) out[lo + n_chosen + i] = hi + i;
+  for (int i = count + tid; i < p.budget; i += kTopkThreads) out[i] = -1;
+  if (tid == 0) p.count_out[unit] = count;
+}
+
 // ============================================================================ host side
 
 namespace {
@@ -692,6 +977,15 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
   tp.chunk = chunk;
   tp.n_mid_pad = plan.n_mid_pad;
   tp.keep_all = plan.keep_all ? 1 : 0;
+  void* targs[] = {&tp};
+  const int free = budget - n_sink - n_recent;
+  if (!plan.keep_all && plan.need_scores && chunk == 1 && plan.n_mid <= kLeanMaxItems && free < plan.n_mid) {
+    const size_t smem = (size_t)align_up(plan.n_mid, 4) * 4;
+    void* fn = reinterpret_cast<void*>(&topk_token_kernel);
+    err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (err != cudaSuccess) return err;
+    return launch_kernel(fn, dim3(units), dim3(kTopkThreads), smem, stream, targs, 0);
+  }
   const int extra = kBins * 4 + kBinCandMax * 8 + 16;      // histogram + boundary-bin candidates
   const int max_items = (kTopkSmemBytes - extra) / 4;
   const int n_items = plan.n_mid;                     // upper bound for chunk mode as well
@@ -700,7 +994,6 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
   err = cudaFuncSetAttribute(reinterpret_cast<void*>(&topk_kernel), cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)smem);
   if (err != cudaSuccess) return err;
-  void* targs[] = {&tp};
   return launch_kernel(reinterpret_cast<void*>(&topk_kernel), dim3(units), dim3(kTopkThreads), smem, stream, targs,
                        0);
 }

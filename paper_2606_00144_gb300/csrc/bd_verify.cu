@@ -7,8 +7,11 @@
 // streams the same number of bytes whatever the batch.  A range covers one or two units;
 // each piece of a unit ("segment") ends in a normalised partial (o, lse), and the last
 // CTA to finish a unit merges its segments (log-sum-exp) into the final bf16 output.
-//   warp 4      TMA producer: 64-key K (and V) tiles, 128-byte swizzle, 3-stage ring,
-//               streaming straight across segment boundaries;
+//   warp 4      TMA producer: 64-key K (and V) tiles, 128-byte swizzle, 5-stage ring,
+//               streaming straight across segment boundaries.  Context rows [0, t_ctx)
+//               are streamed before the grid-dependency wait (they are not written by
+//               the preceding kernel); the wait comes before the first tile that holds
+//               the block's own rows;
 //   warps 0..3  consumers on mma.sync (bd_attn_warp.cuh): the GQA group's packed query
 //               rows are the N side of S^T = K Q^T.
 #include <algorithm>
@@ -22,7 +25,7 @@ namespace bd {
 constexpr int kVKeys = 64;            // keys per pipeline stage
 constexpr int kVConsumers = 4;        // consumer warps
 constexpr int kVThreads = 160;        // + one producer warp
-constexpr int kVStages = 3;
+constexpr int kVStages = 5;
 constexpr int kVMaxSeg = 33;          // bound on the segments of one unit
 
 struct VerifyParams {
@@ -59,8 +62,6 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   constexpr uint32_t HALF_BYTES = kVKeys * 128;
   constexpr int STAGES = kVStages;
 
-  grid_dependency_wait();
-  allow_dependent_launch();
   const int g0 = blockIdx.x * p.tiles_per_cta;
   const int g1 = min(g0 + p.tiles_per_cta, p.total_tiles);
   if (g0 >= g1) return;                           // whole CTA idle
@@ -92,18 +93,24 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
 
   if (warp == kVConsumers) {
     // ------------------------------------------------------------------ producer
+    allow_dependent_launch();
     if (lane == 0) {
       tma_prefetch_map(&kmap);
       if (WITH_V) tma_prefetch_map(&vmap);
       int issued = 0;
+      bool waited = false;
       for (int t = 0; t < ntiles; ++t) {
         const int s = t % STAGES;
         if (t >= STAGES && !mbar_wait(&empty_bar[s], ((t / STAGES) & 1) ^ 1, p.status, abort_flag)) break;
-        uint8_t* st = stage_base + s * L::STAGE_BYTES;
-        mbar_arrive_expect_tx(&full_bar[s], L::STAGE_BYTES);
         const int g = g0 + t;
         const int unit = g / p.tiles_per_unit;
         const int key0 = (g % p.tiles_per_unit) * kVKeys;
+        if (!waited && key0 + kVKeys > p.t_ctx) {      // this tile holds rows of the block itself
+          grid_dependency_wait();
+          waited = true;
+        }
+        uint8_t* st = stage_base + s * L::STAGE_BYTES;
+        mbar_arrive_expect_tx(&full_bar[s], L::STAGE_BYTES);
 #pragma unroll
         for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * HALF_BYTES, &kmap, &full_bar[s], 64 * h, key0, unit);
         if (WITH_V) {
@@ -122,6 +129,8 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   }
 
   // -------------------------------------------------------------------- consumers
+  grid_dependency_wait();                        // the queries come from the preceding kernels
+  allow_dependent_launch();
   const int wq = warp % WQ, wk = warp / WQ;
   const int tig = lane & 3;
   const int nq = p.nq_rows;
