@@ -72,7 +72,8 @@ struct SelectPlan {
   int nq_rows, nq_pad;  // window query rows per KV head (padded to 16)
   int n_mid, n_mid_pad;
   int tiles_per_unit, total_tiles, grid, tiles_per_cta;
-  int stages;
+  int stages;           // K tiles in flight
+  int nqb;              // window-query tile buffers
   int n_acc;            // TMEM accumulators
   uint32_t tmem_cols;
   size_t smem_bytes;

@@ -46,7 +46,7 @@ struct ScoreParams {
   float scale_log2;
 };
 
-template <int D, int STAGES>
+template <int D, int STAGES, int NQB>
 __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p,
                                                              const __grid_constant__ CUtensorMap kmap,
                                                              const __grid_constant__ CUtensorMap qmap) {
@@ -64,8 +64,8 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   const uint32_t qbytes = (uint32_t)p.nq_pad * D * 2;
-  uint8_t* qbuf = smem + kSQOffset;                            // 2 x qbytes
-  uint8_t* kstage = qbuf + 2 * qbytes;                         // STAGES x KTILE (1024-aligned)
+  uint8_t* qbuf = smem + kSQOffset;                            // NQB x qbytes
+  uint8_t* kstage = qbuf + NQB * qbytes;                       // STAGES x KTILE (1024-aligned)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int first = blockIdx.x * p.tiles_per_cta;
@@ -110,12 +110,12 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       const int g = first + i;
       const int unit = g / p.tiles_per_unit, tt = g % p.tiles_per_unit;
       if (unit != cur_unit) {
-        const int qs = qcount & 1;
+        const int qs = qcount % NQB;
         bool ok = true;
         if (lane == 0) {
           // the unit's window-query rows (padded to nq_pad with the next rows, whose scores
           // the epilogue discards) by TMA into the swizzled B-operand tile
-          if (qcount >= 2) ok = mbar_wait(&qempty_bar[qs], ((qcount >> 1) - 1) & 1, p.status, abort_flag);
+          if (qcount >= NQB) ok = mbar_wait(&qempty_bar[qs], ((qcount / NQB) - 1) & 1, p.status, abort_flag);
           if (ok) {
             uint8_t* qb = qbuf + qs * qbytes;
             const uint32_t half_bytes = (uint32_t)p.nq_pad * 128;
@@ -153,11 +153,11 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
         const int unit = g / p.tiles_per_unit;
         const bool last_of_unit = (i == n - 1) || ((g + 1) / p.tiles_per_unit != unit);
         if (unit != cur_unit) {
-          if (!mbar_wait(&qfull_bar[qcount & 1], (qcount >> 1) & 1, p.status, abort_flag)) break;
+          if (!mbar_wait(&qfull_bar[qcount % NQB], (qcount / NQB) & 1, p.status, abort_flag)) break;
           cur_unit = unit;
           ++qcount;
         }
-        const int qs = (qcount - 1) & 1;
+        const int qs = (qcount - 1) % NQB;
         const int s = i % STAGES;
         if (!mbar_wait(&full_bar[s], (i / STAGES) & 1, p.status, abort_flag)) break;
         const int acc = i % n_acc;
@@ -866,12 +866,29 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_token_kernel(const TopkP
 // ============================================================================ host side
 
 namespace {
-constexpr int kSStages = 4;
-void* score_fn(int d) {
-  if (d == 64) return reinterpret_cast<void*>(&score_kernel<64, kSStages>);
-  if (d == 128) return reinterpret_cast<void*>(&score_kernel<128, kSStages>);
-  return nullptr;
+struct ScoreKernel {
+  void* fn;
+  int stages, nqb;
+};
+// Two window-query buffers (a unit switch inside a CTA's range does not stall) and four
+// K stages when they fit, else one Q buffer and as many stages as fit (measured: a fifth
+// stage does not speed the kernel up).
+ScoreKernel score_fn(int d, int nq_pad) {
+  const size_t qbytes = (size_t)nq_pad * d * 2;
+  const size_t kt = (size_t)kSKeys * d * 2;
+  const size_t budget = 227 * 1024 - 1024 - kSQOffset;
+  int stages = 4, nqb = 2;
+  if (2 * qbytes + 4 * kt > budget) {
+    nqb = 1;
+    if (qbytes + 5 * kt <= budget) stages = 5;
+  }
+#define BD_SK(DD, ST, NB) \
+  if (d == DD && stages == ST && nqb == NB) return {reinterpret_cast<void*>(&score_kernel<DD, ST, NB>), ST, NB};
+  BD_SK(64, 5, 1) BD_SK(64, 4, 2) BD_SK(64, 4, 1) BD_SK(128, 5, 1) BD_SK(128, 4, 2) BD_SK(128, 4, 1)
+#undef BD_SK
+  return {nullptr, 0, 0};
 }
+
 uint32_t pow2_at_least(uint32_t x) {
   uint32_t r = 32;
   while (r < x) r <<= 1;
@@ -891,18 +908,21 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   plan->n_mid_pad = (int)align_up(std::max(plan->n_mid, 1), 4);
   const int free = budget - n_sink - n_recent;
   plan->need_scores = !plan->keep_all && plan->n_mid > 0 && free / chunk > 0;
-  if (plan->nq_pad > 256 || !score_fn(s.head_dim)) return false;
+  if (plan->nq_pad > 256) return false;
+  const ScoreKernel sk = score_fn(s.head_dim, plan->nq_pad);
+  if (!sk.fn) return false;
   plan->tiles_per_unit = (plan->n_mid + kSKeys - 1) / kSKeys;
   plan->total_tiles = plan->tiles_per_unit * units;
   plan->grid = std::max(1, std::min(plan->total_tiles, current_sm_count()));
   plan->tiles_per_cta = (plan->total_tiles + plan->grid - 1) / plan->grid;
   plan->grid = std::max(1, (plan->total_tiles + plan->tiles_per_cta - 1) / plan->tiles_per_cta);
-  plan->stages = kSStages;
+  plan->stages = sk.stages;
+  plan->nqb = sk.nqb;
   const uint32_t acc_stride = (uint32_t)align_up(plan->nq_pad, 32);
   plan->n_acc = 4u * acc_stride <= 512u ? 4 : 2;
   plan->tmem_cols = pow2_at_least((uint32_t)plan->n_acc * acc_stride);
-  plan->smem_bytes = 1024 + kSQOffset + 2 * (size_t)plan->nq_pad * s.head_dim * 2 +
-                     (size_t)kSStages * kSKeys * s.head_dim * 2;
+  plan->smem_bytes = 1024 + kSQOffset + (size_t)sk.nqb * plan->nq_pad * s.head_dim * 2 +
+                     (size_t)sk.stages * kSKeys * s.head_dim * 2;
   plan->score_bytes = plan->need_scores ? align_up((size_t)units * plan->n_mid_pad * 4, 256) : 0;
   plan->lse_bytes = align_up((size_t)s.batch * s.h_q * window * 4, 256);
   bd_shape ls = s;
@@ -959,7 +979,7 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
     p.n_acc = plan.n_acc;
     p.tmem_cols = plan.tmem_cols;
     p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
-    void* fn = score_fn(s.head_dim);
+    void* fn = score_fn(s.head_dim, plan.nq_pad).fn;
     err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
     if (err != cudaSuccess) return err;
     void* args[] = {&p, &kmap, &qmap};
