@@ -379,7 +379,8 @@ def gpu_arm(args):
             "unit": "GB/s",
             "frac": round(achieved / peak, 3),
             "bytes_per_launch": verify_launch_bytes,
-            "traffic": None,
+            "traffic": profiled_traffic("verify_kernel", wl.name, ("bd_verify.cu", "bd_attn_warp.cuh", "bd_common.cuh")),
+            "traffic_source": "profiles/verify_kernel_%s.md (ncu dram__bytes_read.sum + dram__bytes_write.sum)" % wl.name,
         },
         "gpu_launches": step.launches_per_step() * args.steps,
         "clocks": clocks,
@@ -408,6 +409,28 @@ def e2e_measure(step, args, world, bytes_per_step):
     return {"value": round(value, 1), "unit": "GB/s", "us_per_step": round(1000.0 * ms / args.steps, 2),
             "h2d_bytes_per_step": io.bytes_in, "d2h_bytes_per_step": io.bytes_out,
             "api": "paper_2606_00144_gb300.SpecStep through the C ABI, pinned host buffers, one CUDA graph"}
+
+
+def profiled_traffic(kernel, workload, sources):
+    """dram bytes read + written per launch from the committed ncu summary, or None when
+    the summary is missing or was taken on other kernel sources than the ones built now."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", f"{kernel}_{workload}.md")
+    try:
+        text = open(path).read()
+    except OSError:
+        return None
+    h = hashlib.sha256()
+    for f in sources:
+        with open(os.path.join(ROOT, "paper_2606_00144_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    fields = dict(ln.split(":", 1) for ln in text.splitlines() if ln.startswith(("source_sha256:", "traffic_bytes")))
+    if fields.get("source_sha256", "").split()[0:1] != [h.hexdigest()[:16]]:
+        return None
+    try:
+        return int(fields["traffic_bytes_per_launch"].strip())
+    except (KeyError, ValueError):
+        return None
 
 
 def measured_hbm_peak():
@@ -497,9 +520,9 @@ def cpu_baseline(wl, budget, n_recent, sel_mode, budget_s=12.0):
     units = n // per_unit
     return {"value": round(nbytes / secs / 1e9, 4), "unit": "GB/s",
             "cores": int(os.environ.get("OMP_NUM_THREADS", "1")), "kind": "oracle",
-            "sample": f"{units} of {wl.batch * wl.h_kv} (sequence, KV head) units of one layer, full step "
-                      f"(selection with carried LSE, {wl.gamma} drafts, verify), numpy fp64; "
-                      f"{secs:.1f} s of oracle time"}
+            "sample": f"{units} (sequence, KV head) unit-steps of one layer, cycling over its "
+                      f"{wl.batch * wl.h_kv} units; each = selection with the carried LSE, {wl.gamma} drafts and "
+                      f"the verify block, numpy fp64; {secs:.1f} s of oracle time"}
 
 
 def reference_arm(args):
