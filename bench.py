@@ -201,7 +201,10 @@ class Step:
         for j in range(self.wl.gamma):
             for l in L:
                 inp = self.layers[l]
-                self.steps[l].draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
+                # the selection of layer l was not written by the kernel just before this one,
+                # except for the first pass of a one-layer step (right after its top-B)
+                ready = j > 0 or self.wl.layers > 1
+                self.steps[l].draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache, view_ready=ready)
         if marks:
             record(marks[2])
         for l in L:

@@ -111,6 +111,15 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
                      int chunk, int32_t* idx_out, int32_t* count_out, void* ws, size_t ws_bytes,
                      void* stream);
 
+/* bd_draft_attn flags. */
+enum {
+  /* idx, count and the context rows [0, t_ctx) of the caches were written before the
+   * kernel that immediately precedes this call on `stream` (true for every pass after the
+   * first of a speculative step): the call may start gathering them while that kernel
+   * finishes.  The queries and the drafted rows are always read after it. */
+  BD_DRAFT_VIEW_READY = 1
+};
+
 /*
  * Drafter decode pass j (0-based) over the sparse view (Algorithm 2, Draft):
  * each query head h of sequence b attends to rows idx[b, g, 0:count[b, g]] and to
@@ -120,12 +129,13 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
  *   idx      int32 [batch, h_kv, budget] positions in [0, t_ctx) (as written by
  *            bd_select_budget; entries past count are ignored); count int32 [batch, h_kv]
  *            with 0 <= count <= budget.
+ *   flags    0 or BD_DRAFT_VIEW_READY.
  *   o_out    bf16 [batch, h_q, d];  lse_out fp32 [batch, h_q] (may be NULL).
  * Constraints: step_j >= 0, t_ctx + step_j < t_cap.
  */
 int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
-                  const int32_t* idx, const int32_t* count, int budget, int step_j, void* o_out,
-                  float* lse_out, void* ws, size_t ws_bytes, void* stream);
+                  const int32_t* idx, const int32_t* count, int budget, int step_j, unsigned flags,
+                  void* o_out, float* lse_out, void* ws, size_t ws_bytes, void* stream);
 
 /*
  * bd_draft_attn without a workspace.  The paper has no counterpart: this entry point
@@ -135,7 +145,7 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
  * must not call cudaMalloc between steps.  Such callers cannot supply the workspace that
  * bd_draft_attn needs.
  *
- * Arguments and results are those of bd_draft_attn, minus ws and ws_bytes.  The call
+ * Arguments and results are those of bd_draft_attn with flags = 0, minus ws and ws_bytes.  The call
  * allocates nothing: its scratch (status word, per-(sequence, KV head) counters and the
  * split-K partials) is a 4 MiB array inside the library's device image, which every GPU
  * that loads the library keeps until the process exits.  A shape whose scratch would not

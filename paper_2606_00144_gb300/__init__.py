@@ -7,6 +7,7 @@ a thin ctypes binding, a step runner and the seeded synthetic workloads.
 """
 
 from .binding import (  # noqa: F401
+    BD_DRAFT_VIEW_READY,
     BD_OP_DRAFT,
     BD_OP_SELECT,
     BD_OP_VERIFY,

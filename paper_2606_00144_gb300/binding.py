@@ -16,6 +16,7 @@ from .build import LIB_PATH
 
 BD_OK = 0
 BD_OP_SELECT, BD_OP_DRAFT, BD_OP_VERIFY = 1, 2, 3
+BD_DRAFT_VIEW_READY = 1
 
 
 class BdShape(ctypes.Structure):
@@ -40,8 +41,8 @@ _SIGNATURES = {
     "bd_workspace_size": (ctypes.c_size_t, [_SHAPE, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "bd_select_budget": (ctypes.c_int, [_SHAPE, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int,
                                         ctypes.c_int, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
-    "bd_draft_attn": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P, _P,
-                                     ctypes.c_size_t, _P]),
+    "bd_draft_attn": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_uint, _P,
+                                     _P, _P, ctypes.c_size_t, _P]),
     "bd_draft_attn_static": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P,
                                             _P]),
     "bd_verify_attn": (ctypes.c_int, [_SHAPE, _P, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
@@ -141,10 +142,10 @@ def bd_select_budget(shape, k_cache, q_window, window_lse, window, budget, n_sin
 
 
 def bd_draft_attn(shape, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
-                  ws: Workspace, stream=None):
+                  ws: Workspace, stream=None, flags=0):
     st = library().bd_draft_attn(ctypes.byref(shape), _ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(idx),
-                                 _ptr(count), int(budget), int(step_j), _ptr(o_out), _ptr(lse_out), ws.ptr,
-                                 ws.nbytes, _stream(stream))
+                                 _ptr(count), int(budget), int(step_j), int(flags), _ptr(o_out), _ptr(lse_out),
+                                 ws.ptr, ws.nbytes, _stream(stream))
     _check("bd_draft_attn", st)
 
 

@@ -192,8 +192,8 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
 }
 
 int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
-                  const int32_t* idx, const int32_t* count, int budget, int step_j, void* o_out, float* lse_out,
-                  void* ws, size_t ws_bytes, void* stream) {
+                  const int32_t* idx, const int32_t* count, int budget, int step_j, unsigned flags, void* o_out,
+                  float* lse_out, void* ws, size_t ws_bytes, void* stream) {
   BD_TRY(check_shape(shape));
   const bd_shape& s = *shape;
   BD_TRY(check_tensor(q, 16));
@@ -204,6 +204,7 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
   BD_TRY(check_tensor(o_out, 16));
   if (lse_out) BD_TRY(check_tensor(lse_out, 4));
   if (budget < 1 || step_j < 0 || (long long)s.t_ctx + step_j >= s.t_cap) return BD_ERR_INVALID_ARG;
+  if (flags & ~BD_DRAFT_VIEW_READY) return BD_ERR_INVALID_ARG;
   if (!group_supported_by_draft(s.h_q / s.h_kv)) return BD_ERR_UNSUPPORTED;
   DraftPlan dp;
   if (!draft_plan(s, budget, step_j + 1, &dp)) return BD_ERR_UNSUPPORTED;
@@ -211,7 +212,7 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
   if (!aligned(ws, 256)) return BD_ERR_MISALIGNED;
   const int units = s.batch * s.h_kv;
   if (ws_bytes < ws_region_offset(units) + draft_partials_bytes(s, dp)) return BD_ERR_WORKSPACE;
-  return map_cuda(launch_draft(s, dp, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
+  return map_cuda(launch_draft(s, dp, q, k_cache, v_cache, idx, count, budget, step_j, flags, o_out, lse_out,
                                region(ws, units), counters(ws), status_word(ws), static_cast<cudaStream_t>(stream)));
 }
 

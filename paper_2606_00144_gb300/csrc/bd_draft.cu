@@ -45,6 +45,7 @@ struct DraftParams {
   int* status;
   int budget, step_j, t_ctx, t_cap, n_split, rows_per_split;
   int n_stage;                 // 1, or 2 when a CTA gathers more than one tile (double buffer)
+  unsigned flags;              // BD_DRAFT_VIEW_READY: gather the selected rows before the dependency wait
   float scale_log2;
 };
 
@@ -66,8 +67,11 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   using L = DraftSmem<D, G>;
   constexpr uint32_t HALF_BYTES = kDRows * 128;
   constexpr int CH = D / 8;                    // 16-byte chunks per row
-  grid_dependency_wait();
-  allow_dependent_launch();
+  const bool early = (p.flags & BD_DRAFT_VIEW_READY) != 0;
+  if (!early) {
+    grid_dependency_wait();
+    allow_dependent_launch();
+  }
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -123,15 +127,18 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
       rowpos[b * kDRows + tid] = pos;
     }
   };
-  auto gather = [&](int tile, int b) {
+  // part 0: context rows (and zero fill), part 1: drafted rows (t_ctx and later), part 2: all
+  auto gather = [&](int tile, int b, int part) {
     const int nrows = min(kDRows, e_end - (e_begin + tile * kDRows));
     uint8_t* kt = stage + b * L::STAGE_BYTES;
     uint8_t* vt = kt + L::TILE_BYTES;
     for (int c = tid; c < kDRows * CH; c += kDThreads) {
       const int r = c / CH, ch = c % CH;
-      const uint32_t off = sw128_offset(r, ch * 8, HALF_BYTES);
       const int pos = rowpos[b * kDRows + r];
       const bool live = r < nrows && pos >= 0;   // others zero-filled (0 * garbage could be NaN in P V)
+      const bool drafted = live && pos >= p.t_ctx;
+      if ((part == 0 && drafted) || (part == 1 && !drafted)) continue;
+      const uint32_t off = sw128_offset(r, ch * 8, HALF_BYTES);
       const size_t src = (size_t)max(pos, 0) * D + ch * 8;
       cp_async16_zfill(kt + off, kunit + src, live);
       cp_async16_zfill(vt + off, vunit + src, live);
@@ -139,22 +146,27 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     cp_async_commit();
   };
 
-  uint32_t bq[1][D / 16][2];
-  WarpAttn<D, 1, true>::load_q(bq, p.q + (size_t)unit * G * D, G, 0, lane);
-  WarpAttn<D, 1, true> wa;
-  wa.init();
   const bool dbuf = p.n_stage == 2;
   if (n_tiles > 0) {
     set_rows(0, 0, true);
     __syncthreads();
-    gather(0, 0);
+    gather(0, 0, early ? 0 : 2);
   }
+  if (early) {   // the selection and the context rows are already in flight
+    grid_dependency_wait();
+    allow_dependent_launch();
+    if (n_tiles > 0) gather(0, 0, 1);
+  }
+  uint32_t bq[1][D / 16][2];
+  WarpAttn<D, 1, true>::load_q(bq, p.q + (size_t)unit * G * D, G, 0, lane);
+  WarpAttn<D, 1, true> wa;
+  wa.init();
   for (int t = 0; t < n_tiles; ++t) {
     const int b = dbuf ? (t & 1) : 0;
     if (dbuf && t + 1 < n_tiles) {
       set_rows(t + 1, (t + 1) & 1, false);
       __syncthreads();
-      gather(t + 1, (t + 1) & 1);
+      gather(t + 1, (t + 1) & 1, 2);
       cp_async_wait<1>();
     } else {
       cp_async_wait<0>();
@@ -174,7 +186,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     if (!dbuf && t + 1 < n_tiles) {
       set_rows(t + 1, 0, false);
       __syncthreads();
-      gather(t + 1, 0);
+      gather(t + 1, 0, 2);
     }
   }
   wa.finish_rows();
@@ -262,8 +274,8 @@ size_t draft_partials_bytes(const bd_shape&, const DraftPlan&) { return 0; }   /
 
 cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q, const void* k_cache,
                          const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
-                         int step_j, void* o_out, float* lse_out, void* ws_region, int* counters,
-                         int* status, cudaStream_t stream) {
+                         int step_j, unsigned flags, void* o_out, float* lse_out, void* ws_region,
+                         int* counters, int* status, cudaStream_t stream) {
   (void)ws_region;
   (void)counters;
   const int units = s.batch * s.h_kv;
@@ -283,6 +295,7 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.n_split = plan.n_split;
   p.rows_per_split = plan.rows_per_split;
   p.n_stage = plan.rows_per_split > kDRows ? 2 : 1;
+  p.flags = flags;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const int g = s.h_q / s.h_kv;
   void* fn = pick(s.head_dim, g);
@@ -341,7 +354,7 @@ cudaError_t launch_draft_static(const bd_shape& s, const DraftPlan& plan, const 
   // arrival counters (they must start at zero) before this call's kernel.
   err = cudaMemsetAsync(b, 0, ws_region_offset(units), stream);
   if (err != cudaSuccess) return err;
-  return launch_draft(s, plan, q, k_cache, v_cache, idx, count, budget, step_j, o_out, lse_out,
+  return launch_draft(s, plan, q, k_cache, v_cache, idx, count, budget, step_j, 0u, o_out, lse_out,
                       b + ws_region_offset(units), reinterpret_cast<int*>(b + ws_counters_offset()),
                       reinterpret_cast<int*>(b), stream);
 }

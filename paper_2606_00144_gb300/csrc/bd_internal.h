@@ -56,8 +56,8 @@ bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan);
 size_t draft_partials_bytes(const bd_shape& s, const DraftPlan& plan);
 cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q, const void* k_cache,
                          const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
-                         int step_j, void* o_out, float* lse_out, void* ws_region, int* counters,
-                         int* status, cudaStream_t stream);
+                         int step_j, unsigned flags, void* o_out, float* lse_out, void* ws_region,
+                         int* counters, int* status, cudaStream_t stream);
 
 // Allocation-free variant: scratch in a file-scope device array of this many bytes.
 size_t draft_static_scratch_bytes();

@@ -39,9 +39,13 @@ class SpecStep:
         B.bd_select_budget(self.shape, k_cache, q_win, window_lse, self.window, self.budget, self.n_sink,
                            self.n_recent, self.chunk, self.idx, self.count, self.ws, stream)
 
-    def draft(self, j, q_j, k_cache, v_cache, stream=None):
+    def draft(self, j, q_j, k_cache, v_cache, stream=None, view_ready=False):
+        """Draft pass j.  view_ready: the selection was not written by the kernel launched
+        just before this one (true for every pass after the first of a step), so the pass may
+        gather the view while that kernel finishes (BD_DRAFT_VIEW_READY)."""
         B.bd_draft_attn(self.shape, q_j, k_cache, v_cache, self.idx, self.count, self.budget, j,
-                        self.draft_o[j], self.draft_lse[j], self.ws, stream)
+                        self.draft_o[j], self.draft_lse[j], self.ws, stream,
+                        flags=B.BD_DRAFT_VIEW_READY if view_ready else 0)
 
     def verify(self, q_verify, k_cache, v_cache, stream=None):
         B.bd_verify_attn(self.shape, q_verify, self.gamma + 1, k_cache, v_cache, self.verify_o,
@@ -50,7 +54,7 @@ class SpecStep:
     def run(self, k_cache, v_cache, q_win, q_draft, q_verify, window_lse=None, stream=None):
         self.select(k_cache, q_win, window_lse, stream)
         for j in range(self.gamma):
-            self.draft(j, q_draft[j], k_cache, v_cache, stream)
+            self.draft(j, q_draft[j], k_cache, v_cache, stream, view_ready=j > 0)
         self.verify(q_verify, k_cache, v_cache, stream)
 
     def window_lse(self, k_cache, q_win, out=None, stream=None):

@@ -57,8 +57,8 @@ def verify(lib, s, q=A, n_q=6, k=A, v=A, o=A, lse=A, ws=A, nbytes=1 << 20):
     return lib.bd_verify_attn(ctypes.byref(s) if s is not None else None, q, n_q, k, v, o, lse, ws, nbytes, None)
 
 
-def draft(lib, s, q=A, k=A, v=A, idx=A, cnt=A, budget=32, j=0, o=A, lse=A, ws=A, nbytes=1 << 20):
-    return lib.bd_draft_attn(ctypes.byref(s), q, k, v, idx, cnt, budget, j, o, lse, ws, nbytes, None)
+def draft(lib, s, q=A, k=A, v=A, idx=A, cnt=A, budget=32, j=0, o=A, lse=A, ws=A, nbytes=1 << 20, flags=0):
+    return lib.bd_draft_attn(ctypes.byref(s), q, k, v, idx, cnt, budget, j, flags, o, lse, ws, nbytes, None)
 
 
 def select(lib, s, k=A, qw=A, lse=A, window=32, budget=40, sink=4, recent=8, chunk=1, idx=A, cnt=A, ws=A,
@@ -89,6 +89,7 @@ def test_draft_validation(lib):
     assert draft(lib, shape(), j=10) == INVALID                       # t_ctx + j >= t_cap
     assert draft(lib, shape(), budget=0) == INVALID
     assert draft(lib, shape(h_q=6, h_kv=2)) == UNSUPPORTED            # group of 3
+    assert draft(lib, shape(), flags=6) == INVALID                    # unknown flag bits
 
 
 def test_select_validation(lib):

@@ -58,7 +58,8 @@ def run_and_check(wl, inp, h, budgets=None, modes=("carry", "self"), chunk=1, ch
         st.idx.copy_(torch.from_numpy(idx_ref).int())
         st.count.copy_(torch.from_numpy(cnt_ref).int())
         for j in range(wl.gamma):
-            st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
+            # passes after the first gather the view before the previous pass has finished
+            st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache, view_ready=j > 0)
             o_ref, l_ref = oracle.draft_attn(h["QD"][j], h["K"], h["V"], idx_ref, cnt_ref, t, j)
             torch.cuda.synchronize()
             stats[f"draft{j}_B{budget}"] = check_attention(st.draft_o[j], st.draft_lse[j], o_ref, l_ref,
