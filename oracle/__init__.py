@@ -1,10 +1,12 @@
 """fp64 CPU oracle (test infrastructure only; never imported by the product path)."""
 
 from .budgetdraft_oracle import (  # noqa: F401
+    accept_greedy,
     attention,
     boundary_score,
     combine,
     draft_attn,
+    greedy_argmax,
     select_budget,
     select_from_scores,
     spec_step,

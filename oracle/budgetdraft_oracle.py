@@ -315,6 +315,56 @@ def spec_step(k_cache, v_cache, q_win, q_draft, q_verify, t_ctx, budget, n_sink,
                 draft_lse=np.stack(dls), verify_o=vo, verify_lse=vl)
 
 
+# ---------------------------------------------------------------------------
+# Greedy acceptance (Eq. accept; Algorithm 2: longest matching prefix, then one
+# verifier token).
+# ---------------------------------------------------------------------------
+
+def greedy_argmax(logits: np.ndarray) -> np.ndarray:
+    """Token ids of the largest logit of every row (the arg max of Eq. accept).
+
+    logits: [rows, vocab].  Ties go to the lowest token id; NaN logits are never
+    chosen; a row with no comparable logit gives id 0.
+    """
+    logits = np.asarray(logits)
+    rows, vocab = logits.shape
+    out = np.zeros(rows, dtype=np.int64)
+    for r in range(rows):
+        best, best_id = None, 0
+        for v in range(vocab):
+            x = logits[r, v]
+            if np.isnan(x):
+                continue
+            if best is None or x > best:
+                best, best_id = x, v
+        out[r] = best_id
+    return out
+
+
+def accept_greedy(draft_tokens: np.ndarray, verify_tokens: np.ndarray):
+    """Accepted length and emitted tokens of one verification (Algorithm 2).
+
+    draft_tokens: [b, gamma] drafter tokens x_hat; verify_tokens: [b, gamma + 1]
+    verifier tokens x_star at the same positions plus one past the block.  k is the
+    largest count with x_hat[i] == x_star[i] for every i < k; the step emits
+    x_hat[0:k] and then x_star[k].  Returns (k [b], emit [b, gamma + 1] padded
+    with -1).
+    """
+    draft_tokens = np.asarray(draft_tokens)
+    verify_tokens = np.asarray(verify_tokens)
+    b, gamma = draft_tokens.shape
+    n = np.zeros(b, dtype=np.int64)
+    emit = np.full((b, gamma + 1), -1, dtype=np.int64)
+    for bi in range(b):
+        k = 0
+        while k < gamma and draft_tokens[bi, k] == verify_tokens[bi, k]:
+            k += 1
+        n[bi] = k
+        emit[bi, :k] = draft_tokens[bi, :k]
+        emit[bi, k] = verify_tokens[bi, k]
+    return n, emit
+
+
 def widen_bf16_bits(bits: np.ndarray) -> np.ndarray:
     """Exact float64 value of bf16 bit patterns (uint16)."""
     bits = np.asarray(bits, dtype=np.uint16).astype(np.uint32) << 16

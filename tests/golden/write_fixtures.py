@@ -74,6 +74,27 @@ FIXTURES = {
         "o": [[1.75, 0.75]],
         "lse": [math.log(4)],
     },
+    "accept_examples.json": {
+        "cite": "Eq. accept and Algorithm 2: accept the longest prefix on which drafter and verifier agree, "
+                "then emit one verifier token",
+        "derivation": "gamma = 4.  Row 0: drafts (7,3,9,2), verifier (7,3,9,2,5): all four agree -> k = 4, emit "
+                      "(7,3,9,2,5).  Row 1: drafts (7,3,9,2), verifier (7,4,9,2,1): first mismatch at index 1 -> "
+                      "k = 1, emit (7,4).  Row 2: verifier (1,...) disagrees at once -> k = 0, emit (1).  Row 3: a "
+                      "later agreement after a mismatch does not count: drafts (5,6,7,8), verifier (5,0,7,8,9) -> "
+                      "k = 1, emit (5,0).",
+        "draft": [[7, 3, 9, 2], [7, 3, 9, 2], [7, 3, 9, 2], [5, 6, 7, 8]],
+        "verify": [[7, 3, 9, 2, 5], [7, 4, 9, 2, 1], [1, 3, 9, 2, 0], [5, 0, 7, 8, 9]],
+        "n_accept": [4, 1, 0, 1],
+        "emit": [[7, 3, 9, 2, 5], [7, 4, -1, -1, -1], [1, -1, -1, -1, -1], [5, 0, -1, -1, -1]],
+    },
+    "argmax_ties.json": {
+        "cite": "Eq. accept: arg max over the vocabulary (reading: ties to the lowest token id, NaN never chosen)",
+        "derivation": "Row 0: maximum 2.5 first at id 1 (also at id 3) -> 1.  Row 1: NaN at id 0 is skipped, max 1.0 at "
+                      "id 2 -> 2.  Row 2: all -inf -> the first id, 0.  Row 3: all NaN -> 0.",
+        "logits": [[0.0, 2.5, -1.0, 2.5], ["nan", 0.5, 1.0, -3.0], ["-inf", "-inf", "-inf", "-inf"],
+                   ["nan", "nan", "nan", "nan"]],
+        "argmax": [1, 2, 0, 0],
+    },
 }
 
 if __name__ == "__main__":

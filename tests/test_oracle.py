@@ -378,3 +378,38 @@ def test_widen_bf16_bits_exact():
     x = torch.randn(1000).to(torch.bfloat16)
     bits = x.view(torch.int16).numpy().view(np.uint16)
     np.testing.assert_array_equal(oracle.widen_bf16_bits(bits), x.double().numpy())
+
+
+# ----------------------------------------------------------------------------- greedy acceptance
+
+def test_golden_accept():
+    fx = load("accept_examples.json")
+    n, emit = oracle.accept_greedy(np.array(fx["draft"]), np.array(fx["verify"]))
+    assert n.tolist() == fx["n_accept"]
+    assert emit.tolist() == fx["emit"]
+
+
+def test_golden_argmax_ties_and_nan():
+    fx = load("argmax_ties.json")
+    logits = np.array([[float(x) for x in row] for row in fx["logits"]])
+    assert oracle.greedy_argmax(logits).tolist() == fx["argmax"]
+
+
+def test_argmax_matches_numpy_without_ties_or_nan():
+    rng = np.random.default_rng(21)
+    x = rng.standard_normal((13, 257))
+    assert np.array_equal(oracle.greedy_argmax(x), np.argmax(x, axis=1))      # numpy: first maximum
+
+
+def test_accept_brute_force():
+    rng = np.random.default_rng(22)
+    for _ in range(200):
+        gamma = int(rng.integers(1, 7))
+        d = rng.integers(0, 3, size=(1, gamma))
+        v = rng.integers(0, 3, size=(1, gamma + 1))
+        n, emit = oracle.accept_greedy(d, v)
+        # brute force: the largest k whose whole prefix agrees
+        k = max(kk for kk in range(gamma + 1) if all(d[0, i] == v[0, i] for i in range(kk)))
+        assert n[0] == k
+        assert emit[0, :k].tolist() == d[0, :k].tolist() and emit[0, k] == v[0, k]
+        assert np.all(emit[0, k + 1:] == -1)
