@@ -323,21 +323,19 @@ def spec_step(k_cache, v_cache, q_win, q_draft, q_verify, t_ctx, budget, n_sink,
 def greedy_argmax(logits: np.ndarray) -> np.ndarray:
     """Token ids of the largest logit of every row (the arg max of Eq. accept).
 
-    logits: [rows, vocab].  Ties go to the lowest token id; NaN logits are never
-    chosen; a row with no comparable logit gives id 0.
+    logits: [rows, vocab], compared in their own type.  Reading: ties go to the lowest
+    token id, NaN logits are never chosen (-0 and +0 compare equal), and a row with no
+    comparable logit gives id 0.
     """
     logits = np.asarray(logits)
-    rows, vocab = logits.shape
+    rows = logits.shape[0]
     out = np.zeros(rows, dtype=np.int64)
     for r in range(rows):
-        best, best_id = None, 0
-        for v in range(vocab):
-            x = logits[r, v]
-            if np.isnan(x):
-                continue
-            if best is None or x > best:
-                best, best_id = x, v
-        out[r] = best_id
+        row = logits[r]
+        comparable = ~np.isnan(row)
+        if comparable.any():
+            top = row[comparable].max()
+            out[r] = int(np.flatnonzero(row == top)[0])      # NaN == top is false
     return out
 
 

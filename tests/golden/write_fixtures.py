@@ -90,10 +90,11 @@ FIXTURES = {
     "argmax_ties.json": {
         "cite": "Eq. accept: arg max over the vocabulary (reading: ties to the lowest token id, NaN never chosen)",
         "derivation": "Row 0: maximum 2.5 first at id 1 (also at id 3) -> 1.  Row 1: NaN at id 0 is skipped, max 1.0 at "
-                      "id 2 -> 2.  Row 2: all -inf -> the first id, 0.  Row 3: all NaN -> 0.",
+                      "id 2 -> 2.  Row 2: all -inf -> the first id, 0.  Row 3: all NaN -> 0.  Row 4: a NaN "
+                      "before -inf values is still skipped -> 1.  Row 5: -0 and +0 are equal -> the first, 1.",
         "logits": [[0.0, 2.5, -1.0, 2.5], ["nan", 0.5, 1.0, -3.0], ["-inf", "-inf", "-inf", "-inf"],
-                   ["nan", "nan", "nan", "nan"]],
-        "argmax": [1, 2, 0, 0],
+                   ["nan", "nan", "nan", "nan"], ["nan", "-inf", "-inf", "nan"], [-1.0, -0.0, 0.0, -2.0]],
+        "argmax": [1, 2, 0, 0, 1, 1],
     },
 }
 

@@ -395,10 +395,23 @@ def test_golden_argmax_ties_and_nan():
     assert oracle.greedy_argmax(logits).tolist() == fx["argmax"]
 
 
-def test_argmax_matches_numpy_without_ties_or_nan():
+def test_argmax_brute_force_with_ties_nan_and_signed_zero():
+    # a plain scan over each row: the first strictly larger comparable value wins
     rng = np.random.default_rng(21)
-    x = rng.standard_normal((13, 257))
-    assert np.array_equal(oracle.greedy_argmax(x), np.argmax(x, axis=1))      # numpy: first maximum
+    x = rng.integers(-3, 4, size=(400, 9)).astype(np.float32)
+    x[rng.random(x.shape) < 0.15] = np.nan
+    x[rng.random(x.shape) < 0.1] = -np.inf
+    x[rng.random(x.shape) < 0.1] = -0.0
+    x[::37] = np.nan
+    x[5::11] = -np.inf                                  # rows whose numbers are all -inf ...
+    x[5::22, ::2] = np.nan                              # ... some behind a leading NaN
+    got = oracle.greedy_argmax(x)
+    for r in range(x.shape[0]):
+        best, best_id = None, 0
+        for v in range(x.shape[1]):
+            if not np.isnan(x[r, v]) and (best is None or x[r, v] > best):
+                best, best_id = x[r, v], v
+        assert got[r] == best_id, r
 
 
 def test_accept_brute_force():
