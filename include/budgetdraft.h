@@ -11,13 +11,19 @@
  *                     causal mask inside the draft block (Algorithm 2, Verify);
  *   bd_combine        the log-sum-exp merge of attention computed over disjoint key
  *                     sets (split-K partials).
+ * and its greedy acceptance in two more:
+ *   bd_argmax         the arg max token of logits rows (Eq. accept);
+ *   bd_accept         the longest agreeing prefix plus the verifier's bonus token
+ *                     (Algorithm 2, accept).
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller; the library
  *     never allocates, frees or keeps a pointer after a call returns.
  *   - bf16 tensors are IEEE bfloat16 (raw 16-bit), fp32 are IEEE float, int32 are
- *     int32_t.  Every tensor is dense row-major in the order written, and every
- *     pointer must be 16-byte aligned.
+ *     int32_t.  Every tensor is dense row-major in the order written.  bf16 tensors
+ *     (caches, queries, outputs) and fp32 split-K partials must be 16-byte aligned;
+ *     other fp32 and int32 tensors 4-byte aligned; logits passed to bd_argmax need
+ *     only their element alignment.
  *   - KV caches are bf16 [batch, h_kv, t_cap, head_dim].  Rows hold post-RoPE keys
  *     and values: position p of (sequence b, KV head g) is row p.  Positions
  *     [0, t_ctx) are the context; rows t_ctx, t_ctx+1, ... hold the tokens of the
@@ -50,7 +56,7 @@ typedef enum bd_status {
   BD_OK = 0,
   BD_ERR_INVALID_ARG = -1,  /* a null pointer, a size out of range, inconsistent shape  */
   BD_ERR_UNSUPPORTED = -2,  /* valid but not implemented (head_dim, too many queries)    */
-  BD_ERR_MISALIGNED = -3,   /* a tensor pointer is not 16-byte aligned                   */
+  BD_ERR_MISALIGNED = -3,   /* a tensor pointer lacks the alignment its call requires    */
   BD_ERR_WORKSPACE = -4,    /* ws is NULL or smaller than bd_workspace_size()            */
   BD_ERR_CUDA = -5,         /* a CUDA runtime call or a launch failed                    */
   BD_ERR_TIMEOUT = -6       /* device side: a bounded wait ran out (status word only)    */
@@ -65,6 +71,9 @@ typedef struct bd_shape {
   int32_t t_ctx;     /* context length T (cached prefix positions)   */
   int32_t t_cap;     /* rows per (sequence, KV head) in the arrays   */
 } bd_shape;
+
+/* Element types of bd_argmax logits. */
+enum { BD_DTYPE_BF16 = 1, BD_DTYPE_F32 = 2 };
 
 /* Operation codes for bd_workspace_size. */
 enum { BD_OP_SELECT = 1, BD_OP_DRAFT = 2, BD_OP_VERIFY = 3 };
@@ -188,6 +197,35 @@ int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_
  */
 int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows, int head_dim,
                void* o_out, float* lse_out, void* stream);
+
+/*
+ * Greedy token choice (Eq. accept: a drafter token is accepted when it equals the
+ * verifier's arg max at the same position): ids_out[r] = arg max over v of
+ * logits[r, v].  Values are compared exactly in the stored type; ties go to the lowest
+ * v, NaN is never chosen, -0 equals +0, and a row without a comparable value (all NaN)
+ * gives 0.
+ *   logits   bf16 or fp32 [rows, vocab] as `dtype` says (BD_DTYPE_*);
+ *   ids_out  int32 [rows].
+ * Constraints: 0 <= rows <= 65535 (0 is a no-op), vocab >= 1.  No workspace.
+ */
+int bd_argmax(const void* logits, int dtype, int rows, int vocab, int32_t* ids_out, void* stream);
+
+/*
+ * Greedy acceptance of one speculative block (Algorithm 2, accept and bonus token):
+ * k = the largest count with draft_tokens[b, i] == verify_tokens[b, i] for every
+ * i < k (0 <= k <= gamma); the step emits draft_tokens[b, 0:k] followed by the
+ * verifier's token verify_tokens[b, k].
+ *   draft_tokens   int32 [batch, gamma]: the drafter's tokens x_hat (may be NULL when
+ *                  gamma == 0);
+ *   verify_tokens  int32 [batch, gamma + 1]: the verifier's arg max at each block
+ *                  position, the last one past the block;
+ *   n_accept_out   int32 [batch]: k (may be NULL);
+ *   emit_out       int32 [batch, gamma + 1]: the k + 1 emitted tokens, then -1 padding
+ *                  (may be NULL, not both).
+ * Constraints: batch >= 0 (0 is a no-op), gamma >= 0.  No workspace.
+ */
+int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* verify_tokens,
+              int32_t* n_accept_out, int32_t* emit_out, void* stream);
 
 /*
  * Reads (and clears) the device status word of a workspace: BD_OK, or the first

@@ -1,19 +1,23 @@
 """GB300 (sm_103a) speculative-step attention of BudgetDraft (arXiv 2606.00144).
 
 The hot path (KV-budget selection, gamma drafter decode passes over the sparse view, the
-verifier's causal block pass and the log-sum-exp merge) lives in libbudgetdraft.so
-(hand-written CUDA, C ABI in include/budgetdraft.h).  This package holds its build step,
+verifier's causal block pass, the log-sum-exp merge and the greedy acceptance) lives in
+libbudgetdraft.so (hand-written CUDA, C ABI in include/budgetdraft.h).  This package holds its build step,
 a thin ctypes binding, a step runner and the seeded synthetic workloads.
 """
 
 from .binding import (  # noqa: F401
     BD_DRAFT_VIEW_READY,
+    BD_DTYPE_BF16,
+    BD_DTYPE_F32,
     BD_OP_DRAFT,
     BD_OP_SELECT,
     BD_OP_VERIFY,
     BdShape,
     BudgetDraftError,
     Workspace,
+    bd_accept,
+    bd_argmax,
     bd_combine,
     bd_draft_attn,
     bd_draft_attn_static,

@@ -17,6 +17,7 @@ from .build import LIB_PATH
 BD_OK = 0
 BD_OP_SELECT, BD_OP_DRAFT, BD_OP_VERIFY = 1, 2, 3
 BD_DRAFT_VIEW_READY = 1
+BD_DTYPE_BF16, BD_DTYPE_F32 = 1, 2
 
 
 class BdShape(ctypes.Structure):
@@ -47,6 +48,8 @@ _SIGNATURES = {
                                             _P]),
     "bd_verify_attn": (ctypes.c_int, [_SHAPE, _P, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "bd_combine": (ctypes.c_int, [_P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P, _P]),
+    "bd_argmax": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P]),
+    "bd_accept": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P]),
     "bd_workspace_status": (ctypes.c_int, [_P, _P]),
     "bd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
 }
@@ -169,6 +172,29 @@ def bd_combine(o_part, lse_part, n_split, rows, head_dim, o_out, lse_out, stream
     st = library().bd_combine(_ptr(o_part), _ptr(lse_part), int(n_split), int(rows), int(head_dim),
                               _ptr(o_out), _ptr(lse_out), _stream(stream))
     _check("bd_combine", st)
+
+
+def bd_argmax(logits, ids_out, stream=None):
+    """ids_out[r] = arg max of logits[r] (bf16 or fp32 [rows, vocab], int32 [rows])."""
+    if logits.dtype == torch.bfloat16:
+        dtype = BD_DTYPE_BF16
+    elif logits.dtype == torch.float32:
+        dtype = BD_DTYPE_F32
+    else:
+        raise TypeError(f"bd_argmax: logits must be bf16 or fp32, got {logits.dtype}")
+    if logits.dim() != 2 or not logits.is_contiguous():
+        raise ValueError("bd_argmax: logits must be a contiguous [rows, vocab] tensor")
+    rows, vocab = logits.shape
+    st = library().bd_argmax(_ptr(logits), dtype, int(rows), int(vocab), _ptr(ids_out), _stream(stream))
+    _check("bd_argmax", st)
+
+
+def bd_accept(draft_tokens, verify_tokens, n_accept_out, emit_out, stream=None):
+    """Accepted prefix length and emitted tokens (int32 [batch, gamma], [batch, gamma + 1])."""
+    batch, g1 = verify_tokens.shape
+    st = library().bd_accept(int(batch), int(g1 - 1), _ptr(draft_tokens), _ptr(verify_tokens), _ptr(n_accept_out),
+                             _ptr(emit_out), _stream(stream))
+    _check("bd_accept", st)
 
 
 def bd_workspace_status(ws: Workspace, stream=None) -> int:

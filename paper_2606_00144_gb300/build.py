@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(BUILD_DIR, "libbudgetdraft.so")
-SOURCES = ("bd_api.cu", "bd_verify.cu", "bd_draft.cu", "bd_select.cu", "bd_combine.cu")
+SOURCES = ("bd_api.cu", "bd_verify.cu", "bd_draft.cu", "bd_select.cu", "bd_combine.cu", "bd_accept.cu")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
                 "-I", INCLUDE]

@@ -280,6 +280,31 @@ int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows
                                  static_cast<cudaStream_t>(stream)));
 }
 
+int bd_argmax(const void* logits, int dtype, int rows, int vocab, int32_t* ids_out, void* stream) {
+  if (dtype != BD_DTYPE_BF16 && dtype != BD_DTYPE_F32) return BD_ERR_INVALID_ARG;
+  if (rows < 0 || vocab < 1) return BD_ERR_INVALID_ARG;
+  if (rows == 0) return BD_OK;
+  if (rows > 65535) return BD_ERR_UNSUPPORTED;
+  BD_TRY(check_tensor(logits, dtype == BD_DTYPE_BF16 ? 2 : 4));
+  BD_TRY(check_tensor(ids_out, 4));
+  return map_cuda(launch_argmax(logits, dtype == BD_DTYPE_BF16, rows, vocab, ids_out,
+                                static_cast<cudaStream_t>(stream)));
+}
+
+int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* verify_tokens,
+              int32_t* n_accept_out, int32_t* emit_out, void* stream) {
+  if (batch < 0 || gamma < 0) return BD_ERR_INVALID_ARG;
+  if (batch == 0) return BD_OK;
+  if ((long long)batch * (gamma + 1) >= (1LL << 31)) return BD_ERR_UNSUPPORTED;
+  if (gamma > 0) BD_TRY(check_tensor(draft_tokens, 4));
+  BD_TRY(check_tensor(verify_tokens, 4));
+  if (!n_accept_out && !emit_out) return BD_ERR_INVALID_ARG;
+  if (n_accept_out) BD_TRY(check_tensor(n_accept_out, 4));
+  if (emit_out) BD_TRY(check_tensor(emit_out, 4));
+  return map_cuda(launch_accept(batch, gamma, draft_tokens, verify_tokens, n_accept_out, emit_out,
+                                static_cast<cudaStream_t>(stream)));
+}
+
 int bd_workspace_status(void* ws, void* stream) {
   if (!ws) return BD_ERR_INVALID_ARG;
   int host = 0;

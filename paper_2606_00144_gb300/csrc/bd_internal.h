@@ -93,6 +93,13 @@ cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_spl
                            int head_dim, void* o_out, float* lse_out, cudaStream_t stream);
 int combine_rows_per_block(int n_split);
 
+// ---------------------------------------------------------------------------- acceptance
+int argmax_cluster(int rows, int vocab);   // CTAs per row
+cudaError_t launch_argmax(const void* logits, bool bf16, int rows, int vocab, int32_t* ids_out,
+                          cudaStream_t stream);
+cudaError_t launch_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* verify_tokens,
+                          int32_t* n_accept, int32_t* emit, cudaStream_t stream);
+
 // ---------------------------------------------------------------------------- TMA maps
 // 3-D map over a [units, rows_total (stride t_cap), head_dim] bf16 cache: only rows
 // [0, n_rows) of each unit are addressable (the rest reads as zero).  Box = 64 columns x

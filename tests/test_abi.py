@@ -122,3 +122,29 @@ def test_product_path_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(binding, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError):
         binding.library()
+
+
+def test_argmax_validation(lib):
+    f = lib.bd_argmax
+    assert f(A, 3, 4, 100, A, None) == INVALID                         # unknown dtype
+    assert f(A, binding.BD_DTYPE_BF16, -1, 100, A, None) == INVALID
+    assert f(A, binding.BD_DTYPE_BF16, 4, 0, A, None) == INVALID
+    assert f(A, binding.BD_DTYPE_BF16, 0, 100, A, None) == BD_OK         # empty: no-op
+    assert f(A, binding.BD_DTYPE_BF16, 70000, 100, A, None) == UNSUPPORTED
+    assert f(A + 1, binding.BD_DTYPE_BF16, 4, 100, A, None) == MISALIGNED
+    assert f(A + 2, binding.BD_DTYPE_F32, 4, 100, A, None) == MISALIGNED
+    assert f(A, binding.BD_DTYPE_F32, 4, 100, A + 2, None) == MISALIGNED
+    assert f(A, binding.BD_DTYPE_F32, 4, 100, None, None) == INVALID
+    assert f(None, binding.BD_DTYPE_F32, 4, 100, A, None) == INVALID
+
+
+def test_accept_validation(lib):
+    f = lib.bd_accept
+    assert f(-1, 5, A, A, A, A, None) == INVALID
+    assert f(8, -1, A, A, A, A, None) == INVALID
+    assert f(0, 5, None, None, None, None, None) == BD_OK               # empty: no-op
+    assert f(8, 5, A, A, None, None, None) == INVALID                    # nothing to write
+    assert f(8, 5, None, A, A, A, None) == INVALID                       # drafts needed when gamma > 0
+    assert f(8, 5, A, None, A, A, None) == INVALID
+    assert f(8, 5, A, A, A + 2, A, None) == MISALIGNED
+    assert f(8, 5, A, A, A, A + 1, None) == MISALIGNED
