@@ -48,15 +48,16 @@ FALLBACK_HBM_GBS = 6800.0
 
 # ----------------------------------------------------------------------------- bytes the method must read
 
-def step_bytes(wl, budget, n_recent, sel_mode):
+def step_bytes(wl, budget, n_recent, sel_mode, n_sink=None):
     """Algorithmic HBM bytes of one step on one layer, by phase."""
     row = wl.head_dim * 2
     units = wl.batch * wl.h_kv
     t = wl.t_ctx
+    sink = wl.n_sink if n_sink is None else n_sink
     if budget >= t:
         sel = 0
     else:
-        sel = (t - wl.n_sink - n_recent) * row * units          # middle keys, once
+        sel = (t - sink - n_recent) * row * units               # middle keys, once
         if sel_mode == "self":
             sel += t * row * units                               # window LSE over the prefix
     draft = (min(budget, t) + wl.gamma) * 2 * row * units       # sparse view once + drafted rows
@@ -167,14 +168,21 @@ def record(ev_pair):
 # ----------------------------------------------------------------------------- the GPU arm
 
 class Step:
-    """All layers of one workload: inputs, carried window LSE, one SpecStep per layer."""
+    """All layers of one workload: inputs, carried window LSE, one SpecStep per layer.
 
-    def __init__(self, wl, budget, n_recent, sel_mode, device):
+    `share`: another Step whose inputs and carried LSE this one reuses (a policy variant on
+    the same data)."""
+
+    def __init__(self, wl, budget, n_recent, sel_mode, device, share=None, n_sink=None, chunk=1):
         import paper_2606_00144_gb300 as bd
         self.wl, self.budget, self.n_recent, self.sel_mode = wl, budget, n_recent, sel_mode
+        self.n_sink = wl.n_sink if n_sink is None else n_sink
+        self.steps = [bd.SpecStep(wl.batch, wl.h_q, wl.h_kv, wl.head_dim, wl.t_ctx, wl.t_cap, budget, self.n_sink,
+                                  n_recent, wl.window, wl.gamma, chunk, device) for _ in range(wl.layers)]
+        if share is not None:
+            self.layers, self.lse = share.layers, share.lse
+            return
         self.layers = [W.make_layer(wl, l, device) for l in range(wl.layers)]
-        self.steps = [bd.SpecStep.for_workload(wl, budget=budget, n_recent=n_recent, device=device)
-                      for _ in range(wl.layers)]
         self.lse = []
         for st, inp in zip(self.steps, self.layers):
             # carried state: the window rows' LSE as the verify kernel leaves it
@@ -189,13 +197,16 @@ class Step:
             sel = 2 + (1 if self.sel_mode == "self" else 0)
         return self.wl.layers * (sel + self.wl.gamma + 1)
 
-    def run(self, marks=None):
-        """One step; marks = [select, draft, verify, end] timing events (or None)."""
+    def run(self, marks=None, select=True):
+        """One step; marks = [select, draft, verify, end] timing events (or None).  With
+        select=False the sparse views of the last selection are reused (selection amortised
+        over steps, as Algorithm 2 sparsifies once at prefill)."""
         L = range(self.wl.layers)
         if marks:
             record(marks[0])
-        for l in L:
-            self.steps[l].select(self.layers[l].k_cache, self.layers[l].q_win, self.lse[l])
+        if select:
+            for l in L:
+                self.steps[l].select(self.layers[l].k_cache, self.layers[l].q_win, self.lse[l])
         if marks:
             record(marks[1])
         for j in range(self.wl.gamma):
@@ -203,7 +214,7 @@ class Step:
                 inp = self.layers[l]
                 # the selection of layer l was not written by the kernel just before this one,
                 # except for the first pass of a one-layer step (right after its top-B)
-                ready = j > 0 or self.wl.layers > 1
+                ready = j > 0 or self.wl.layers > 1 or not select
                 self.steps[l].draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache, view_ready=ready)
         if marks:
             record(marks[2])
@@ -390,6 +401,8 @@ def gpu_arm(args):
     }
     if not args.no_e2e:
         line["e2e"] = e2e_measure(step, args, world, layer_bytes["total"])
+    if world == 1 and not args.no_extras:
+        line["extras"] = extras(step, args)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget, n_recent, args.sel_mode, budget_s=args.cpu_seconds)
     if rank == 0:
@@ -397,6 +410,94 @@ def gpu_arm(args):
     if world > 1:
         import torch.distributed as dist
         dist.destroy_process_group()
+
+
+def time_per_step(fn, n_steps, graph_steps):
+    """µs per call of fn, captured graph_steps calls per CUDA graph (CUDA events)."""
+    S = graph_len(n_steps, graph_steps)
+    fn()
+    torch.cuda.synchronize()
+    g = capture(lambda i: fn(), S)
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    ms = timed_replays([g] * (n_steps // S), 1)
+    return 1000.0 * ms / n_steps
+
+
+VOCAB = 128256        # Llama-3 vocabulary (the logits rows the acceptance reads)
+
+
+def extras(step, args):
+    """Measurements of the steps beside the headline path (not part of `value`):
+    selection amortised over steps, the greedy acceptance, and the paper's chunk policy."""
+    import paper_2606_00144_gb300 as bd
+    wl = step.wl
+    n = args.extra_steps
+    gs = args.graph_steps
+    out = {}
+
+    # drafts + verify only: the sparse views of one selection reused (Algorithm 2 sparsifies at prefill)
+    per = step_bytes(wl, step.budget, step.n_recent, step.sel_mode)
+    us = time_per_step(lambda: step.run(select=False), n, gs)
+    b = (per["draft"] + per["verify"]) * wl.layers
+    out["amortized_step"] = {"us_per_step": round(us, 2), "GB/s": round(b / (us * 1e-6) / 1e9, 1),
+                             "bytes_per_step": b, "launches_per_step": wl.layers * (wl.gamma + 1)}
+
+    # greedy acceptance (Eq. accept, Algorithm 2): arg max of every drafter pass and of the
+    # verify block over a Llama-3 vocabulary, then the prefix test; synthetic bf16 logits
+    gen = torch.Generator(device="cuda").manual_seed(wl.seed + 77)
+    dl = torch.randn(wl.gamma, wl.batch, VOCAB, device="cuda", generator=gen).to(torch.bfloat16)
+    vl = torch.randn(wl.batch, wl.gamma + 1, VOCAB, device="cuda", generator=gen).to(torch.bfloat16)
+    d_ids = torch.empty(wl.gamma, wl.batch, dtype=torch.int32, device="cuda")
+    v_ids = torch.empty(wl.batch, wl.gamma + 1, dtype=torch.int32, device="cuda")
+    n_acc = torch.empty(wl.batch, dtype=torch.int32, device="cuda")
+    emit = torch.empty(wl.batch, wl.gamma + 1, dtype=torch.int32, device="cuda")
+
+    def accept():
+        for j in range(wl.gamma):
+            bd.bd_argmax(dl[j], d_ids[j])
+        bd.bd_argmax(vl.view(-1, VOCAB), v_ids.view(-1))
+        bd.bd_accept(d_ids, v_ids, n_acc, emit)
+
+    def step_with_accept():
+        # the step in its dependency order: each drafter pass is followed by its token choice
+        L = range(wl.layers)
+        for l in L:
+            step.steps[l].select(step.layers[l].k_cache, step.layers[l].q_win, step.lse[l])
+        for j in range(wl.gamma):
+            for l in L:
+                inp = step.layers[l]
+                step.steps[l].draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache, view_ready=j > 0 or wl.layers > 1)
+            bd.bd_argmax(dl[j], d_ids[j])
+        for l in L:
+            inp = step.layers[l]
+            step.steps[l].verify(inp.q_verify, inp.k_cache, inp.v_cache)
+        bd.bd_argmax(vl.view(-1, VOCAB), v_ids.view(-1))
+        bd.bd_accept(d_ids, v_ids, n_acc, emit)
+
+    us_acc = time_per_step(accept, n, gs)
+    us_full = time_per_step(step_with_accept, n, gs)
+    lb = (dl.numel() + vl.numel()) * 2
+    out["accept"] = {"vocab": VOCAB, "us_per_step": round(us_acc, 2), "logits_bytes": lb,
+                     "GB/s": round(lb / (us_acc * 1e-6) / 1e9, 1), "launches_per_step": wl.gamma + 2,
+                     "step_with_accept_us": round(us_full, 2)}
+
+    # the paper's chunk policy (Sec. 3.4, s = 8): same sink/recent/budget, and the pure
+    # top-floor(B/s)-chunks form with no sink or recent window over a budget sweep
+    if step.budget < wl.t_ctx:
+        rows = []
+        cases = [(step.budget, wl.n_sink, step.n_recent)] + [(bb, 0, 0) for bb in (256, 512, 1024, 2048)]
+        for bb, sink, rec in cases:
+            v = Step(wl, bb, rec, step.sel_mode, "cuda", share=step, n_sink=sink, chunk=8)
+            us = time_per_step(v.run, n, gs)
+            pb = step_bytes(wl, bb, rec, step.sel_mode, n_sink=sink)["total"] * wl.layers
+            rows.append({"budget": bb, "n_sink": sink, "n_recent": rec, "chunk": 8, "us_per_step": round(us, 2),
+                         "GB/s": round(pb / (us * 1e-6) / 1e9, 1)})
+            del v
+        out["chunk_policy"] = rows
+    out["note"] = "each timed over %d graphed steps outside the headline timed region" % n
+    return out
 
 
 def e2e_measure(step, args, world, bytes_per_step):
@@ -583,6 +684,8 @@ def parse():
     p.add_argument("--cpu-seconds", type=float, default=12.0)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--no-extras", action="store_true", help="skip the amortised / acceptance / chunk-policy lines")
+    p.add_argument("--extra-steps", type=int, default=500)
     a = p.parse_args()
     if a.warmup < 3:
         p.error("--warmup must be >= 3")

@@ -212,11 +212,12 @@ int bd_argmax(const void* logits, int dtype, int rows, int vocab, int32_t* ids_o
 
 /*
  * Greedy acceptance of one speculative block (Algorithm 2, accept and bonus token):
- * k = the largest count with draft_tokens[b, i] == verify_tokens[b, i] for every
- * i < k (0 <= k <= gamma); the step emits draft_tokens[b, 0:k] followed by the
+ * k = the largest count with draft_tokens[i, b] == verify_tokens[b, i] for every
+ * i < k (0 <= k <= gamma); the step emits those k drafter tokens followed by the
  * verifier's token verify_tokens[b, k].
- *   draft_tokens   int32 [batch, gamma]: the drafter's tokens x_hat (may be NULL when
- *                  gamma == 0);
+ *   draft_tokens   int32 [gamma, batch]: the drafter's tokens x_hat, pass-major (row j
+ *                  holds pass j's token of every sequence, as bd_argmax writes them one
+ *                  pass at a time); may be NULL when gamma == 0;
  *   verify_tokens  int32 [batch, gamma + 1]: the verifier's arg max at each block
  *                  position, the last one past the block;
  *   n_accept_out   int32 [batch]: k (may be NULL);

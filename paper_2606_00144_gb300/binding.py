@@ -190,7 +190,8 @@ def bd_argmax(logits, ids_out, stream=None):
 
 
 def bd_accept(draft_tokens, verify_tokens, n_accept_out, emit_out, stream=None):
-    """Accepted prefix length and emitted tokens (int32 [batch, gamma], [batch, gamma + 1])."""
+    """Accepted prefix length and emitted tokens: draft_tokens int32 [gamma, batch] (pass-major),
+    verify_tokens int32 [batch, gamma + 1]."""
     batch, g1 = verify_tokens.shape
     st = library().bd_accept(int(batch), int(g1 - 1), _ptr(draft_tokens), _ptr(verify_tokens), _ptr(n_accept_out),
                              _ptr(emit_out), _stream(stream))

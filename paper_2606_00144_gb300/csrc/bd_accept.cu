@@ -190,7 +190,8 @@ __global__ void __launch_bounds__(kAThreads) argmax_kernel(const void* logits, i
 }
 
 // One thread per sequence: k = the number of leading positions where drafter and verifier
-// agree; emit x_hat[0:k], then the verifier's token x_star[k] (the bonus), then -1 padding.
+// agree; emit x_hat[0:k] (equal to x_star[0:k]), then the verifier's token x_star[k] (the
+// bonus), then -1 padding.
 __global__ void __launch_bounds__(128) accept_kernel(int batch, int gamma, const int32_t* draft_tokens,
                                                      const int32_t* verify_tokens, int32_t* n_accept,
                                                      int32_t* emit) {
@@ -198,14 +199,15 @@ __global__ void __launch_bounds__(128) accept_kernel(int batch, int gamma, const
   allow_dependent_launch();
   const int b = blockIdx.x * blockDim.x + threadIdx.x;
   if (b >= batch) return;
-  const int32_t* d = draft_tokens + (size_t)b * gamma;
+  // draft_tokens is pass-major: pass j's token of sequence b sits at [j, b]
+  const int32_t* d = draft_tokens + b;
   const int32_t* v = verify_tokens + (size_t)b * (gamma + 1);
   int k = 0;
-  while (k < gamma && d[k] == v[k]) ++k;
+  while (k < gamma && d[(size_t)k * batch] == v[k]) ++k;
   if (n_accept) n_accept[b] = k;
   if (emit) {
     int32_t* e = emit + (size_t)b * (gamma + 1);
-    for (int i = 0; i <= gamma; ++i) e[i] = i < k ? d[i] : (i == k ? v[k] : -1);
+    for (int i = 0; i <= gamma; ++i) e[i] = i < k ? v[i] : (i == k ? v[k] : -1);
   }
 }
 

@@ -106,7 +106,7 @@ def test_accept_matches_oracle(batch, gamma):
     d, v = token_blocks(batch, gamma, seed=batch * 31 + gamma)
     n = torch.full((batch,), -7, dtype=torch.int32, device="cuda")
     emit = torch.full((batch, gamma + 1), -7, dtype=torch.int32, device="cuda")
-    dd = torch.from_numpy(d).cuda() if gamma > 0 else None
+    dd = torch.from_numpy(np.ascontiguousarray(d.T)).cuda() if gamma > 0 else None   # pass-major
     bd.bd_accept(dd, torch.from_numpy(v).cuda(), n, emit)
     torch.cuda.synchronize()
     n_ref, emit_ref = oracle.accept_greedy(d, v)
@@ -132,7 +132,7 @@ def test_accept_from_logits_pipeline():
     bd.bd_argmax(vl.view(batch * (gamma + 1), vocab), v_ids.view(-1))
     n = torch.empty(batch, dtype=torch.int32, device="cuda")
     emit = torch.empty(batch, gamma + 1, dtype=torch.int32, device="cuda")
-    bd.bd_accept(d_ids.t().contiguous(), v_ids, n, emit)
+    bd.bd_accept(d_ids, v_ids, n, emit)
     torch.cuda.synchronize()
     d_ref = oracle.greedy_argmax(draft_logits.float().numpy().reshape(-1, vocab)).reshape(gamma, batch).T
     v_ref = oracle.greedy_argmax(verify_logits.float().numpy().reshape(-1, vocab)).reshape(batch, gamma + 1)

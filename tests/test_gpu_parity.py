@@ -5,6 +5,8 @@ Covers the five evaluation workloads (the 32-layer stack on whole and sampled la
 partial tail, the degenerate cases, the standalone merge and determinism.
 """
 
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -28,8 +30,11 @@ def host(inp):
                 QV=f64(inp.q_verify))
 
 
-def run_and_check(wl, inp, h, budgets=None, modes=("carry", "self"), chunk=1, check_steps=True, tag=""):
-    """Runs selection (both modes), gamma drafts on the oracle's selection, and verify."""
+def run_and_check(wl, inp, h, budgets=None, modes=("carry", "self"), chunk=1, check_steps=True, tag="",
+                  recent=None):
+    """Runs selection (both modes), gamma drafts on the oracle's selection, and verify.
+    recent: the recent window of every budget (default: the workload's for its own budget,
+    budget // 4 for the others)."""
     t = wl.t_ctx
     lse_ref = oracle.window_lse(h["QW"], h["K"], t)
     score_ref = oracle.window_scores(h["QW"], h["K"], lse_ref, t)
@@ -37,7 +42,7 @@ def run_and_check(wl, inp, h, budgets=None, modes=("carry", "self"), chunk=1, ch
     stats = {}
     budgets = budgets or [wl.budget]
     for budget in budgets:
-        n_recent = wl.n_recent if budget == wl.budget else budget // 4
+        n_recent = recent if recent is not None else (wl.n_recent if budget == wl.budget else budget // 4)
         st = bd.SpecStep.for_workload(wl, budget=budget, n_recent=n_recent, chunk=chunk)
         idx_ref = np.full((wl.batch, wl.h_kv, budget), -1)
         cnt_ref = np.zeros((wl.batch, wl.h_kv), dtype=np.int64)
@@ -97,6 +102,19 @@ def test_l8b_16k_b8_budget_sweep():
     wl = W.WORKLOADS["l8b_16k_b8"]
     inp = W.make_layer(wl, 0, "cuda")
     run_and_check(wl, inp, host(inp), budgets=list(W.SWEEP_16K), modes=("carry",), tag="l8b_16k_b8")
+
+
+def test_l8b_16k_b8_chunk_policy():
+    """The paper's policy (Sec. 3.4): the top floor(B/8) chunks of 8 by cumulative attention
+    with no sink or recent window, over the budget sweep; then s = 8 beside the default
+    sink and recent window."""
+    wl = W.WORKLOADS["l8b_16k_b8"]
+    inp = W.make_layer(wl, 0, "cuda")
+    h = host(inp)
+    pure = dataclasses.replace(wl, n_sink=0, n_recent=0)
+    run_and_check(pure, inp, h, budgets=[512, 256, 1024, 2048], chunk=8, recent=0, modes=("carry",),
+                  tag="chunk8 pure")
+    run_and_check(wl, inp, h, chunk=8, modes=("carry", "self"), check_steps=False, tag="chunk8")
 
 
 def test_l8b_16k_b8_self_mode_selection():
