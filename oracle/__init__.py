@@ -2,7 +2,10 @@
 
 from .budgetdraft_oracle import (  # noqa: F401
     accept_greedy,
+    advance_window,
+    append_view,
     attention,
+    batch_advance,
     boundary_score,
     combine,
     draft_attn,

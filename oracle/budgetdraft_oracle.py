@@ -22,7 +22,7 @@ Paper references (BudgetDraft, arXiv 2606.00144):
   * Cache update: accepted tokens are appended to both caches (Algorithm 2,
     Update), which is why the drafter's own new rows join its sparse view.
 
-Readings where the paper is silent (each is listed in the design doc):
+Readings where the paper is silent:
   * softmax scale 1/sqrt(d), no soft-cap; caches hold post-RoPE keys, so a row
     gathered by index keeps its position (Sec. 3.4, explicit position IDs);
   * "cumulative attention weight" of key k = sum over the GQA group's heads and
@@ -361,6 +361,61 @@ def accept_greedy(draft_tokens: np.ndarray, verify_tokens: np.ndarray):
         emit[bi, :k] = draft_tokens[bi, :k]
         emit[bi, k] = verify_tokens[bi, k]
     return n, emit
+
+
+# ---------------------------------------------------------------------------
+# Cache update after acceptance (Algorithm 2, Update): the accepted block rows join
+# the context, the observation window slides over them, and the drafter's sparse
+# view takes the accepted positions.
+# ---------------------------------------------------------------------------
+
+def batch_advance(n_accept: np.ndarray, n_q: int) -> int:
+    """Positions every sequence of a batch that shares one context length advances by.
+
+    Reading (the paper treats one sequence): sequence b keeps its block rows
+    t_ctx .. t_ctx + n_accept[b] (the rows whose tokens are now settled: the token the
+    block started from and the accepted drafts); a batch stored with one common length
+    advances by the smallest of these counts, so every sequence stays on tokens its
+    verifier has confirmed.
+    """
+    k = int(np.min(np.asarray(n_accept))) if np.asarray(n_accept).size else 0
+    return min(max(k, 0), n_q - 1) + 1
+
+
+def advance_window(q_win: np.ndarray, lse_win: np.ndarray, q_verify: np.ndarray,
+                   lse_verify: np.ndarray, advance: int):
+    """Slides the observation window by `advance` positions over the verified block.
+
+    q_win [b, h_q, W, d] and lse_win [b, h_q, W] hold the queries and softmax
+    normalisers of positions t_ctx - W .. t_ctx - 1; q_verify [b, h_q, n_q, d] and
+    lse_verify [b, h_q, n_q] those of the block positions t_ctx .. t_ctx + n_q - 1.
+    Returns the same arrays for positions t_ctx + advance - W .. t_ctx + advance - 1.
+    """
+    W = q_win.shape[2]
+    q_all = np.concatenate([q_win, q_verify[:, :, :advance]], axis=2)
+    l_all = np.concatenate([lse_win, lse_verify[:, :, :advance]], axis=2)
+    return q_all[:, :, advance: advance + W].copy(), l_all[:, :, advance: advance + W].copy()
+
+
+def append_view(idx: np.ndarray, count: np.ndarray, t_ctx: int, advance: int, capacity: int):
+    """The sparse view after the settled block rows t_ctx .. t_ctx + advance - 1 join it.
+
+    idx [b, h_kv, capacity] (ascending positions, -1 padding), count [b, h_kv].
+    Returns new (idx, count); a view without room for the new rows is returned
+    unchanged and flagged in the third result.
+    """
+    idx = np.array(idx, copy=True)
+    count = np.array(count, copy=True)
+    full = False
+    for b in range(idx.shape[0]):
+        for g in range(idx.shape[1]):
+            c = int(count[b, g])
+            if c + advance > capacity:
+                full = True
+                continue
+            idx[b, g, c: c + advance] = np.arange(t_ctx, t_ctx + advance)
+            count[b, g] = c + advance
+    return idx, count, full
 
 
 def widen_bf16_bits(bits: np.ndarray) -> np.ndarray:

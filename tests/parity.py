@@ -1,6 +1,6 @@
 """Comparison helpers for the CUDA path against the fp64 oracle.
 
-Tolerances ("Parity bar"):
+Tolerances:
   * attention outputs (bf16 inputs, fp32 accumulation, bf16 output):
       max-abs  max |o_gpu - o_ref|                     <= 1e-2
       max-rel  max over rows of max_d |o_gpu - o_ref| / max_d |o_ref|   <= 1e-2

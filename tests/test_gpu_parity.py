@@ -318,6 +318,22 @@ def test_combine_merges_disjoint_draft_views():
     check_attention(out, lse, o_ref, l_ref, "combine of draft parts")
 
 
+@pytest.mark.parametrize("planted", [0, 100])
+def test_tied_scores_take_lowest_positions(planted):
+    """Middle keys set to zero have exactly equal scores: all of them (planted = 0: min = max)
+    or all but every planted-th key, with the boundary falling among the ties in a bin too
+    crowded to rank, so the exact radix select runs (split over a cluster of CTAs)."""
+    wl = W.tiny_workload(batch=1, h_q=8, h_kv=2, head_dim=128, t_ctx=6000, budget=300, n_sink=4, n_recent=32,
+                         window=32, gamma=1)
+    inp = W.make_layer(wl, 0, "cuda")
+    mid = inp.k_cache[:, :, wl.n_sink: wl.t_ctx - wl.n_recent]
+    keep = mid[:, :, ::planted].clone() if planted else None
+    mid.zero_()
+    if planted:
+        mid[:, :, ::planted] = keep
+    run_and_check(wl, inp, host(inp), check_steps=False, tag=f"ties planted={planted}")
+
+
 def test_determinism():
     wl = W.WORKLOADS["l8b_4k"]
     inp = W.make_layer(wl, 0, "cuda")

@@ -426,3 +426,39 @@ def test_accept_brute_force():
         assert n[0] == k
         assert emit[0, :k].tolist() == d[0, :k].tolist() and emit[0, k] == v[0, k]
         assert np.all(emit[0, k + 1:] == -1)
+
+
+# ----------------------------------------------------------------------------- cache update
+
+def test_batch_advance_closed_cases():
+    assert oracle.batch_advance(np.array([3, 1, 4]), n_q=6) == 2       # smallest k = 1 -> k + 1 rows
+    assert oracle.batch_advance(np.array([5, 5]), n_q=6) == 6          # all drafts accepted
+    assert oracle.batch_advance(np.array([0, 5]), n_q=6) == 1          # only the starting token settles
+    assert oracle.batch_advance(np.array([9]), n_q=6) == 6             # clamped to the block
+
+
+@pytest.mark.parametrize("window,advance", [(8, 3), (8, 6), (2, 3)])
+def test_advance_window_equals_window_of_the_longer_context(window, advance):
+    # the slid window must hold exactly the queries and causal LSEs a window taken at the
+    # new length would have: compare with window_lse recomputed from scratch there
+    rng = np.random.default_rng(31)
+    b, hq, hkv, d, t, n_q = 2, 4, 2, 16, 40, 6
+    K = rng.standard_normal((b, hkv, t + n_q, d))
+    q_all = rng.standard_normal((b, hq, t + n_q, d))
+    q_win = q_all[:, :, t - window: t]
+    lse_win = oracle.window_lse(q_win, K, t)
+    q_ver = q_all[:, :, t: t + n_q]
+    _, lse_ver = oracle.verify_attn(q_ver, K, K, t)
+    q_new, lse_new = oracle.advance_window(q_win, lse_win, q_ver, lse_ver, advance)
+    t2 = t + advance
+    assert np.array_equal(q_new, q_all[:, :, t2 - window: t2])
+    np.testing.assert_allclose(lse_new, oracle.window_lse(q_all[:, :, t2 - window: t2], K, t2), rtol=0, atol=1e-12)
+
+
+def test_append_view_closed_example():
+    idx = np.array([[[0, 5, 9, -1, -1, -1]]])
+    cnt = np.array([[3]])
+    i2, c2, full = oracle.append_view(idx, cnt, t_ctx=12, advance=2, capacity=6)
+    assert i2.tolist() == [[[0, 5, 9, 12, 13, -1]]] and c2.tolist() == [[5]] and not full
+    i3, c3, full = oracle.append_view(i2, c2, t_ctx=14, advance=2, capacity=6)
+    assert i3.tolist() == i2.tolist() and c3.tolist() == [[5]] and full     # no room: unchanged
