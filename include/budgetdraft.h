@@ -14,7 +14,10 @@
  * and its greedy acceptance in two more:
  *   bd_argmax         the arg max token of logits rows (Eq. accept);
  *   bd_accept         the longest agreeing prefix plus the verifier's bonus token
- *                     (Algorithm 2, accept).
+ *                     (Algorithm 2, accept);
+ * and the cache update after it in one more:
+ *   bd_advance        slides the observation window over the settled block rows and
+ *                     appends their positions to the sparse view (Algorithm 2, Update).
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller; the library
@@ -227,6 +230,36 @@ int bd_argmax(const void* logits, int dtype, int rows, int vocab, int32_t* ids_o
  */
 int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* verify_tokens,
               int32_t* n_accept_out, int32_t* emit_out, void* stream);
+
+/*
+ * Cache update after acceptance (Algorithm 2, Update).  The verify block held positions
+ * t_ctx .. t_ctx + n_q - 1 (the token the step started from, then the drafts); after
+ * acceptance of k_b drafts, sequence b's rows t_ctx .. t_ctx + k_b are settled.  One call
+ * shares one context length over the batch, so the batch advances by
+ *     a = min_b(clamp(n_accept[b], 0, n_q - 1)) + 1
+ * positions (every sequence stays on tokens its verifier confirmed).  The K/V rows of the
+ * block were written into the caches before bd_verify_attn and stay where they are: the
+ * caller makes the settled ones context by using t_ctx + a as the next step's t_ctx.
+ * This call updates the state that carry-mode selection and the drafter need:
+ *   - q_window / window_lse slide by a: they hold positions t_ctx + a - W ..
+ *     t_ctx + a - 1 afterwards, the new rows taken from q_verify / verify_lse (the
+ *     verifier's softmax normaliser of a block row IS that row's causal window LSE);
+ *   - idx / count (optional): positions t_ctx .. t_ctx + a - 1 are appended to every
+ *     unit's view (Algorithm 2 appends accepted tokens to the sparse cache); a unit
+ *     whose view has no room (count + a > idx_capacity) is left unchanged.
+ *   n_accept      int32 [batch] accepted drafts per sequence (bd_accept's n_accept_out);
+ *   q_verify      bf16 [batch, h_q, n_q, d]; verify_lse fp32 [batch, h_q, n_q] (NULL
+ *                 together with window_lse);
+ *   q_window      bf16 [batch, h_q, window, d], window_lse fp32 [batch, h_q, window]:
+ *                 read and rewritten in place;
+ *   idx           int32 [batch, h_kv, idx_capacity], count int32 [batch, h_kv] (both
+ *                 NULL to skip the view);
+ *   advance_out   int32 [1]: a (may be NULL).
+ * Constraints: 1 <= window <= t_ctx, 1 <= n_q, t_ctx + n_q <= t_cap.  No workspace.
+ */
+int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_accept, const void* q_verify,
+               const float* verify_lse, void* q_window, float* window_lse, int32_t* idx, int32_t* count,
+               int idx_capacity, int32_t* advance_out, void* stream);
 
 /*
  * Reads (and clears) the device status word of a workspace: BD_OK, or the first

@@ -17,6 +17,7 @@ from .binding import (  # noqa: F401
     BudgetDraftError,
     Workspace,
     bd_accept,
+    bd_advance,
     bd_argmax,
     bd_combine,
     bd_draft_attn,

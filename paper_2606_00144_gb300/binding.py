@@ -50,6 +50,8 @@ _SIGNATURES = {
     "bd_combine": (ctypes.c_int, [_P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P, _P]),
     "bd_argmax": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P]),
     "bd_accept": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P]),
+    "bd_advance": (ctypes.c_int, [_SHAPE, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int, _P,
+                                  _P]),
     "bd_workspace_status": (ctypes.c_int, [_P, _P]),
     "bd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
 }
@@ -196,6 +198,16 @@ def bd_accept(draft_tokens, verify_tokens, n_accept_out, emit_out, stream=None):
     st = library().bd_accept(int(batch), int(g1 - 1), _ptr(draft_tokens), _ptr(verify_tokens), _ptr(n_accept_out),
                              _ptr(emit_out), _stream(stream))
     _check("bd_accept", st)
+
+
+def bd_advance(shape, window, n_q, n_accept, q_verify, verify_lse, q_window, window_lse, idx=None, count=None,
+               advance_out=None, stream=None):
+    """Slides the observation window (and appends to the sparse view) after acceptance."""
+    cap = int(idx.shape[-1]) if idx is not None else 0
+    st = library().bd_advance(ctypes.byref(shape), int(window), int(n_q), _ptr(n_accept), _ptr(q_verify),
+                              _ptr(verify_lse), _ptr(q_window), _ptr(window_lse), _ptr(idx), _ptr(count), cap,
+                              _ptr(advance_out), _stream(stream))
+    _check("bd_advance", st)
 
 
 def bd_workspace_status(ws: Workspace, stream=None) -> int:

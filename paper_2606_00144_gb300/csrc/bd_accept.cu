@@ -1,6 +1,8 @@
 // Greedy acceptance of a speculative step (Eq. accept; Algorithm 2, accept and bonus
 // token): the arg max of every logits row (bd_argmax), then the longest prefix on which the
-// drafter's and the verifier's tokens agree plus one verifier token (bd_accept).
+// drafter's and the verifier's tokens agree plus one verifier token (bd_accept); and the
+// cache update that follows (Algorithm 2, Update; bd_advance): the observation window
+// slides over the settled block rows and the drafter's sparse view takes their positions.
 //
 // bd_argmax is a plain streaming reduction: each row is split across a cluster of up to 8
 // CTAs; every thread reads batches of 16-byte vectors, takes each batch's maximum with
@@ -11,6 +13,7 @@
 #include <cooperative_groups.h>
 
 #include <algorithm>
+#include <climits>
 
 #include "bd_common.cuh"
 #include "bd_internal.h"
@@ -209,6 +212,107 @@ __global__ void __launch_bounds__(128) accept_kernel(int batch, int gamma, const
     int32_t* e = emit + (size_t)b * (gamma + 1);
     for (int i = 0; i <= gamma; ++i) e[i] = i < k ? v[i] : (i == k ? v[k] : -1);
   }
+}
+
+// ---------------------------------------------------------------------------- bd_advance
+constexpr int kVThreads = 128;
+
+struct AdvanceParams {
+  const int32_t* n_accept;        // [batch]
+  const __nv_bfloat16* q_verify;  // [batch, h_q, n_q, D]
+  const float* lse_verify;        // [batch, h_q, n_q] or null
+  __nv_bfloat16* q_win;           // [batch, h_q, window, D], slid in place
+  float* lse_win;                 // [batch, h_q, window] or null
+  int32_t* idx;                   // [batch, h_kv, capacity] or null
+  int32_t* count;                 // [batch, h_kv]
+  int32_t* advance_out;           // [1] or null
+  int batch, h_q, h_kv, window, n_q, t_ctx, capacity;
+};
+
+// grid (h_q, batch).  CTA (h, b) slides the window of query head h of sequence b: new row w
+// is old row w + a while that exists, else block row w + a - window.  The new rows are
+// staged in shared memory before any is written, so the slide is done in place.  CTAs with
+// h < h_kv also append the positions t_ctx .. t_ctx + a - 1 to the view of unit (b, h).
+template <int D>
+__global__ void __launch_bounds__(kVThreads) advance_kernel(const AdvanceParams p) {
+  extern __shared__ __align__(16) uint8_t adv_smem[];
+  __shared__ int s_min[kVThreads / 32];
+  grid_dependency_wait();
+  allow_dependent_launch();
+  const int tid = threadIdx.x, h = blockIdx.x, b = blockIdx.y;
+  int m = INT_MAX;
+  for (int i = tid; i < p.batch; i += kVThreads) m = min(m, p.n_accept[i]);
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) m = min(m, __shfl_xor_sync(0xffffffffu, m, off));
+  if ((tid & 31) == 0) s_min[tid >> 5] = m;
+  __syncthreads();
+  m = s_min[0];
+#pragma unroll
+  for (int w = 1; w < kVThreads / 32; ++w) m = min(m, s_min[w]);
+  const int a = min(max(m, 0), p.n_q - 1) + 1;       // settled rows: the start token + k accepted
+  if (h == 0 && b == 0 && tid == 0 && p.advance_out) p.advance_out[0] = a;
+
+  const int W = p.window;
+  constexpr int CH = D / 8;                         // 16-byte chunks per row
+  uint4* qs = reinterpret_cast<uint4*>(adv_smem);   // [W][CH]
+  float* ls = reinterpret_cast<float*>(qs + (size_t)W * CH);
+  const size_t bh = (size_t)b * p.h_q + h;
+  const uint4* qw = reinterpret_cast<const uint4*>(p.q_win + bh * W * D);
+  const uint4* qv = reinterpret_cast<const uint4*>(p.q_verify + bh * p.n_q * D);
+  for (int i = tid; i < W * CH; i += kVThreads) {
+    const int w = i / CH, c = i % CH, src = w + a;
+    qs[i] = src < W ? qw[(size_t)src * CH + c] : qv[(size_t)(src - W) * CH + c];
+  }
+  if (p.lse_win) {
+    for (int w = tid; w < W; w += kVThreads) {
+      const int src = w + a;
+      ls[w] = src < W ? p.lse_win[bh * W + src] : p.lse_verify[bh * p.n_q + src - W];
+    }
+  }
+  __syncthreads();
+  uint4* qo = reinterpret_cast<uint4*>(p.q_win + bh * W * D);
+  for (int i = tid; i < W * CH; i += kVThreads) qo[i] = qs[i];
+  if (p.lse_win)
+    for (int w = tid; w < W; w += kVThreads) p.lse_win[bh * W + w] = ls[w];
+
+  if (p.idx && h < p.h_kv) {
+    const size_t u = (size_t)b * p.h_kv + h;
+    const int c = p.count[u];
+    if (c + a <= p.capacity) {                      // a view without room is left as it is
+      for (int i = tid; i < a; i += kVThreads) p.idx[u * p.capacity + c + i] = p.t_ctx + i;
+      __syncthreads();
+      if (tid == 0) p.count[u] = c + a;
+    }
+  }
+}
+
+size_t advance_smem(int window, int head_dim) { return (size_t)window * head_dim * 2 + (size_t)window * 4; }
+
+cudaError_t launch_advance(const bd_shape& s, int window, int n_q, const int32_t* n_accept, const void* q_verify,
+                           const float* verify_lse, void* q_window, float* window_lse, int32_t* idx, int32_t* count,
+                           int capacity, int32_t* advance_out, cudaStream_t stream) {
+  AdvanceParams p;
+  p.n_accept = n_accept;
+  p.q_verify = static_cast<const __nv_bfloat16*>(q_verify);
+  p.lse_verify = verify_lse;
+  p.q_win = static_cast<__nv_bfloat16*>(q_window);
+  p.lse_win = window_lse;
+  p.idx = idx;
+  p.count = count;
+  p.advance_out = advance_out;
+  p.batch = s.batch;
+  p.h_q = s.h_q;
+  p.h_kv = s.h_kv;
+  p.window = window;
+  p.n_q = n_q;
+  p.t_ctx = s.t_ctx;
+  p.capacity = capacity;
+  const size_t smem = advance_smem(window, s.head_dim);
+  void* fn = s.head_dim == 64 ? reinterpret_cast<void*>(&advance_kernel<64>) : reinterpret_cast<void*>(&advance_kernel<128>);
+  cudaError_t err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (err != cudaSuccess) return err;
+  void* args[] = {&p};
+  return launch_kernel(fn, dim3(s.h_q, s.batch), dim3(kVThreads), smem, stream, args, 0);
 }
 
 int argmax_cluster(int rows, int vocab) {

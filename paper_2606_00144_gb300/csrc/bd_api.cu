@@ -305,6 +305,33 @@ int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* 
                                 static_cast<cudaStream_t>(stream)));
 }
 
+int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_accept, const void* q_verify,
+               const float* verify_lse, void* q_window, float* window_lse, int32_t* idx, int32_t* count,
+               int idx_capacity, int32_t* advance_out, void* stream) {
+  BD_TRY(check_shape(shape));
+  const bd_shape& s = *shape;
+  if (window < 1 || window > s.t_ctx || n_q < 1 || s.t_ctx + n_q > s.t_cap) return BD_ERR_INVALID_ARG;
+  if ((verify_lse == nullptr) != (window_lse == nullptr)) return BD_ERR_INVALID_ARG;
+  if ((idx == nullptr) != (count == nullptr)) return BD_ERR_INVALID_ARG;
+  if (idx && idx_capacity < 1) return BD_ERR_INVALID_ARG;
+  if (s.batch > 65535 || s.h_q > 65535) return BD_ERR_UNSUPPORTED;
+  if (advance_smem(window, s.head_dim) > 200 * 1024) return BD_ERR_UNSUPPORTED;
+  BD_TRY(check_tensor(n_accept, 4));
+  BD_TRY(check_tensor(q_verify, 16));
+  BD_TRY(check_tensor(q_window, 16));
+  if (window_lse) {
+    BD_TRY(check_tensor(verify_lse, 4));
+    BD_TRY(check_tensor(window_lse, 4));
+  }
+  if (idx) {
+    BD_TRY(check_tensor(idx, 4));
+    BD_TRY(check_tensor(count, 4));
+  }
+  if (advance_out) BD_TRY(check_tensor(advance_out, 4));
+  return map_cuda(launch_advance(s, window, n_q, n_accept, q_verify, verify_lse, q_window, window_lse, idx, count,
+                                 idx_capacity, advance_out, static_cast<cudaStream_t>(stream)));
+}
+
 int bd_workspace_status(void* ws, void* stream) {
   if (!ws) return BD_ERR_INVALID_ARG;
   int host = 0;

@@ -99,6 +99,10 @@ cudaError_t launch_argmax(const void* logits, bool bf16, int rows, int vocab, in
                           cudaStream_t stream);
 cudaError_t launch_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* verify_tokens,
                           int32_t* n_accept, int32_t* emit, cudaStream_t stream);
+size_t advance_smem(int window, int head_dim);
+cudaError_t launch_advance(const bd_shape& s, int window, int n_q, const int32_t* n_accept, const void* q_verify,
+                           const float* verify_lse, void* q_window, float* window_lse, int32_t* idx, int32_t* count,
+                           int capacity, int32_t* advance_out, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------- TMA maps
 // 3-D map over a [units, rows_total (stride t_cap), head_dim] bf16 cache: only rows

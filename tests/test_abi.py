@@ -148,3 +148,18 @@ def test_accept_validation(lib):
     assert f(8, 5, A, None, A, A, None) == INVALID
     assert f(8, 5, A, A, A + 2, A, None) == MISALIGNED
     assert f(8, 5, A, A, A, A + 1, None) == MISALIGNED
+
+
+def test_advance_validation(lib):
+    def adv(s, window=32, n_q=6, n_acc=A, qv=A, lv=A, qw=A, lw=A, idx=A, cnt=A, cap=64, out=A):
+        return lib.bd_advance(ctypes.byref(s), window, n_q, n_acc, qv, lv, qw, lw, idx, cnt, cap, out, None)
+    assert adv(shape(), window=0) == INVALID
+    assert adv(shape(), window=101) == INVALID                          # window > t_ctx
+    assert adv(shape(), n_q=11) == INVALID                              # t_ctx + n_q > t_cap
+    assert adv(shape(), lv=None) == INVALID                             # lse ring needs both sides
+    assert adv(shape(), cnt=None) == INVALID                            # view needs idx and count
+    assert adv(shape(), cap=0) == INVALID
+    assert adv(shape(), n_acc=None) == INVALID
+    assert adv(shape(), qw=A + 8) == MISALIGNED
+    assert adv(shape(), out=A + 2) == MISALIGNED
+    assert adv(shape(head_dim=96)) == UNSUPPORTED
