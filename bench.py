@@ -131,12 +131,20 @@ def dist_env():
 
 
 def max_over_ranks(x, world):
+    """The largest x over the ranks (the slowest rank's time)."""
     if world == 1:
         return x
     import torch.distributed as dist
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def job_throughput(bytes_per_step_per_rank, steps, world, ms_max):
+    """Whole-job GB/s: every rank runs its own replica of the step (weak scaling), so the
+    job moves world x the per-rank bytes in the slowest rank's time."""
+    return bytes_per_step_per_rank * steps * world / (ms_max / 1e3) / 1e9
 
 
 def barrier(world):
@@ -350,8 +358,7 @@ def gpu_arm(args):
 
     ms_per_step = ms / args.steps
     us = 1000.0 * ms_per_step
-    total_bytes = layer_bytes["total"] * args.steps * world
-    value = total_bytes / (ms / 1e3) / 1e9
+    value = job_throughput(layer_bytes["total"], args.steps, world, ms)
     peak, peak_src = measured_hbm_peak()
     verify_launch_bytes = per["verify"]
     verify_us = phase_us["verify"] / wl.layers
@@ -509,7 +516,7 @@ def e2e_measure(step, args, world, bytes_per_step):
     torch.cuda.synchronize()
     ms = timed_replays([g] * (args.steps // S), world)
     ms = max_over_ranks(ms, world)
-    value = bytes_per_step * args.steps * world / (ms / 1e3) / 1e9
+    value = job_throughput(bytes_per_step, args.steps, world, ms)
     return {"value": round(value, 1), "unit": "GB/s", "us_per_step": round(1000.0 * ms / args.steps, 2),
             "h2d_bytes_per_step": io.bytes_in, "d2h_bytes_per_step": io.bytes_out,
             "api": "paper_2606_00144_gb300.SpecStep through the C ABI, pinned host buffers, one CUDA graph"}
