@@ -278,32 +278,52 @@ template <int D, typename RowMap>
 __device__ __forceinline__ void merge_partials(const float* o_part, const float* lse_part, int n_split,
                                                int rows, size_t split_stride, size_t lse_split_stride,
                                                __nv_bfloat16* o_out, float* lse_out, RowMap out_row,
-                                               float* w_smem, int tid, int nthreads, int bar_id) {
-  // weights exp(lse_s - L) per (split, row)
+                                               float* w_smem, int tid, int nthreads, int bar_id,
+                                               float* stage = nullptr, size_t stage_floats = 0) {
+  constexpr int D4 = D / 4;
+  const int total = rows * D4;
+  // The parts were written by other CTAs just before and sit in L2: latency, not bandwidth,
+  // decides this merge.  With a staging area big enough, every part row is copied into
+  // shared memory by cp.async while the lse loads are in flight too: one round trip.
+  const bool staged = o_out != nullptr && stage != nullptr && (size_t)n_split * rows * D <= stage_floats;
+  if (staged) {
+    for (int i = tid; i < n_split * total; i += nthreads) {
+      const int sp = i / total, j = i % total;
+      const int r = j / D4, c = (j % D4) * 4;
+      cp_async16(stage + (size_t)i * 4, o_part + sp * split_stride + (size_t)r * D + c);
+    }
+    cp_async_commit();
+  }
+  // weights exp(lse_s - L) per (split, row); a row's lse values are all requested at once
   for (int r = tid; r < rows; r += nthreads) {
     float mx = -INFINITY;
-    for (int s = 0; s < n_split; ++s) mx = fmaxf(mx, __ldcg(lse_part + s * lse_split_stride + r));
+#pragma unroll 8
+    for (int sp = 0; sp < n_split; ++sp) {
+      const float l = __ldcg(lse_part + sp * lse_split_stride + r);
+      w_smem[sp * rows + r] = l;
+      mx = fmaxf(mx, l);
+    }
     float tot = 0.f;
-    for (int s = 0; s < n_split; ++s) {
-      const float l = __ldcg(lse_part + s * lse_split_stride + r);
-      const float w = (mx == -INFINITY) ? 0.f : fast_exp2((l - mx) * kLog2e);
-      w_smem[s * rows + r] = w;
+    for (int sp = 0; sp < n_split; ++sp) {
+      const float w = (mx == -INFINITY) ? 0.f : fast_exp2((w_smem[sp * rows + r] - mx) * kLog2e);
+      w_smem[sp * rows + r] = w;
       tot += w;
     }
     const float inv = tot > 0.f ? 1.f / tot : 0.f;
-    for (int s = 0; s < n_split; ++s) w_smem[s * rows + r] *= inv;
+    for (int sp = 0; sp < n_split; ++sp) w_smem[sp * rows + r] *= inv;
     if (lse_out) lse_out[out_row(r)] = (mx == -INFINITY) ? -INFINITY : mx + logf(tot);
   }
+  if (staged) cp_async_wait<0>();
   named_bar(bar_id, nthreads);
   if (o_out == nullptr) return;
-  constexpr int D4 = D / 4;
-  for (int i = tid; i < rows * D4; i += nthreads) {
+  for (int i = tid; i < total; i += nthreads) {
     const int r = i / D4, c = (i % D4) * 4;
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-    for (int s = 0; s < n_split; ++s) {
-      const float w = w_smem[s * rows + r];
+    for (int sp = 0; sp < n_split; ++sp) {
+      const float w = w_smem[sp * rows + r];
       if (w != 0.f) {
-        const float4 v = __ldcg(reinterpret_cast<const float4*>(o_part + s * split_stride + (size_t)r * D + c));
+        const float4 v = staged ? *reinterpret_cast<const float4*>(stage + ((size_t)sp * total + i) * 4)
+                                : __ldcg(reinterpret_cast<const float4*>(o_part + sp * split_stride + (size_t)r * D + c));
         acc.x += w * v.x;
         acc.y += w * v.y;
         acc.z += w * v.z;

@@ -199,7 +199,7 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
         const size_t base = (size_t)unit * p.max_seg;
         merge_partials<D>(p.o_part + base * nq * D, p.lse_part + base * nq, n_seg, nq, (size_t)nq * D, (size_t)nq,
                           WITH_V ? p.o + row0 * D : nullptr, p.lse ? p.lse + row0 : nullptr, [](int r) { return r; },
-                          w_s, tid, NCT, 1);
+                          w_s, tid, NCT, 1, m_s, L::kMerge / 4);
         if (tid == 0) p.counters[unit] = 0;
       }
     }
