@@ -32,7 +32,8 @@ struct VerifyPlan {
   int nt, wq;           // n-tiles per warp, warp groups along queries
   int tiles_per_unit;   // 64-key tiles over [0, t_ctx + n_q)
   int total_tiles;      // over all units
-  int tiles_per_cta;    // contiguous range of the global tile list per CTA
+  int tiles_per_cta;    // contiguous range of the virtual tile list per CTA
+  int seg_cost;         // virtual tiles before each unit's tiles (the cost of starting a unit)
   int grid;
   int max_seg;          // most CTAs that share one unit
   int stages;

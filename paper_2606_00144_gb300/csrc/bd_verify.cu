@@ -36,9 +36,26 @@ struct VerifyParams {
   float* lse_part;     // [units][max_seg][nq_rows]
   int* counters;       // [units]
   int* status;
-  int n_q, nq_rows, t_ctx, tiles_per_unit, total_tiles, tiles_per_cta, max_seg;
+  int n_q, nq_rows, t_ctx, tiles_per_unit, total_tiles, max_seg;
+  int seg_cost;        // virtual tiles charged for each unit a CTA starts (see verify_plan)
+  int vtiles_per_cta;  // contiguous range of the virtual tile list per CTA
   float scale_log2;    // log2(e) / sqrt(D)
 };
+
+// The global tile list is cut into equal CTA ranges after every unit's tiles are preceded
+// by `seg_cost` virtual tiles: a CTA whose range starts a unit (and so stops to merge one
+// segment and load new queries) receives that many fewer real tiles.  Virtual index v of
+// unit u = v / (tpu + a) maps to the unit's first real tile while inside its virtual prefix.
+__host__ __device__ __forceinline__ int real_tile(int v, int tpu, int a) {
+  const int u = v / (tpu + a);
+  const int r = v - u * (tpu + a);
+  return u * tpu + (r > a ? r - a : 0);
+}
+// The CTA whose range holds real tile g.
+__host__ __device__ __forceinline__ int tile_owner(int g, int tpu, int a, int vtpc) {
+  const int u = g / tpu;
+  return (u * (tpu + a) + a + (g - u * tpu)) / vtpc;
+}
 
 template <int D, int NT, int WQ, bool WITH_V>
 struct VerifySmem {
@@ -62,8 +79,10 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   constexpr uint32_t HALF_BYTES = kVKeys * 128;
   constexpr int STAGES = kVStages;
 
-  const int g0 = blockIdx.x * p.tiles_per_cta;
-  const int g1 = min(g0 + p.tiles_per_cta, p.total_tiles);
+  const int n_units = p.total_tiles / p.tiles_per_unit;
+  const int v_end = n_units * (p.tiles_per_unit + p.seg_cost);
+  const int g0 = real_tile(blockIdx.x * p.vtiles_per_cta, p.tiles_per_unit, p.seg_cost);
+  const int g1 = real_tile(min((blockIdx.x + 1) * p.vtiles_per_cta, v_end), p.tiles_per_unit, p.seg_cost);
   if (g0 >= g1) return;                           // whole CTA idle
   const int ntiles = g1 - g0;
 
@@ -178,8 +197,8 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     wa.store(m_s, l_s, o_s, wk, NQC, wq * NT, lane);
     named_bar(1, NCT);
     const int c = blockIdx.x;
-    const int c_first = (unit * p.tiles_per_unit) / p.tiles_per_cta;
-    const int c_last = ((unit + 1) * p.tiles_per_unit - 1) / p.tiles_per_cta;
+    const int c_first = tile_owner(unit * p.tiles_per_unit, p.tiles_per_unit, p.seg_cost, p.vtiles_per_cta);
+    const int c_last = tile_owner((unit + 1) * p.tiles_per_unit - 1, p.tiles_per_unit, p.seg_cost, p.vtiles_per_cta);
     const int n_seg = c_last - c_first + 1;
     const size_t row0 = (size_t)unit * nq;
     if (n_seg == 1) {
@@ -290,14 +309,31 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   const long n_keys = (long)s.t_ctx + n_q;
   plan->tiles_per_unit = (int)((n_keys + kVKeys - 1) / kVKeys);
   const long units = (long)s.batch * s.h_kv;
-  const long total = units * plan->tiles_per_unit;
+  const int tpu = plan->tiles_per_unit;
+  const long total = units * tpu;
   const long ctas = std::max(1, current_sm_count() * occupancy(k));
-  long tpc = (total + ctas - 1) / ctas;
-  tpc = std::max<long>(tpc, (plan->tiles_per_unit + kVMaxSeg - 2) / (kVMaxSeg - 1));   // <= kVMaxSeg segments
-  plan->tiles_per_cta = (int)tpc;
+  // A segment end (merge of the warps' partials, its write, the arrival, the next unit's
+  // queries) costs about 3 us of streaming time; charge it as virtual tiles at the rate
+  // one CTA streams at when every SM streams (measured ~6.5 TB/s over all SMs).
+  const double tile_bytes = (double)kVKeys * s.head_dim * 2 * (with_v ? 2 : 1);
+  const double tile_us = tile_bytes / (6.5e6 / (double)std::max(1, current_sm_count()));
+  const int a = (int)std::min(16.0, std::max(0.0, 3.0 / tile_us + 0.5));
+  const long vtotal = units * (tpu + a);
+  if (vtotal >= (1L << 31)) return false;
+  long vtpc = (vtotal + ctas - 1) / ctas;
+  vtpc = std::max<long>(vtpc, (tpu + a + kVMaxSeg - 2) / (kVMaxSeg - 1));   // <= kVMaxSeg segments
+  plan->seg_cost = a;
+  plan->tiles_per_cta = (int)vtpc;
   plan->total_tiles = (int)total;
-  plan->grid = (int)((total + tpc - 1) / tpc);
-  plan->max_seg = (int)std::min<long>(kVMaxSeg, (plan->tiles_per_unit + tpc - 1) / tpc + 1);
+  plan->grid = (int)((vtotal + vtpc - 1) / vtpc);
+  int max_seg = 1;
+  for (long u = 0; u < units; ++u) {
+    const int c0 = tile_owner((int)(u * tpu), tpu, a, (int)vtpc);
+    const int c1 = tile_owner((int)(u * tpu + tpu - 1), tpu, a, (int)vtpc);
+    max_seg = std::max(max_seg, c1 - c0 + 1);
+  }
+  if (max_seg > kVMaxSeg) return false;
+  plan->max_seg = max_seg;
   return true;
 }
 
@@ -334,7 +370,8 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.t_ctx = s.t_ctx;
   p.tiles_per_unit = plan.tiles_per_unit;
   p.total_tiles = plan.total_tiles;
-  p.tiles_per_cta = plan.tiles_per_cta;
+  p.seg_cost = plan.seg_cost;
+  p.vtiles_per_cta = plan.tiles_per_cta;
   p.max_seg = plan.max_seg;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const KernelInfo k = select_kernel(s.head_dim, plan.nt, plan.wq, plan.with_v);
