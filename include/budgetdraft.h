@@ -15,7 +15,8 @@
  *   bd_argmax         the arg max token of logits rows (Eq. accept);
  *   bd_accept         the longest agreeing prefix plus the verifier's bonus token
  *                     (Algorithm 2, accept);
- * and the cache update after it in one more:
+ * and the cache update around it in two more:
+ *   bd_write_block_rows  writes the block's new K/V rows into the caches;
  *   bd_advance        slides the observation window over the settled block rows and
  *                     appends their positions to the sparse view (Algorithm 2, Update).
  *
@@ -260,6 +261,18 @@ int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* 
 int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_accept, const void* q_verify,
                const float* verify_lse, void* q_window, float* window_lse, int32_t* idx, int32_t* count,
                int idx_capacity, int32_t* advance_out, void* stream);
+
+/*
+ * Writes the K/V rows of the current block into the caches: rows t_ctx .. t_ctx + n_rows - 1
+ * of every (sequence, KV head) (Algorithm 2, Update: new tokens' keys and values join the
+ * cache).  Two strided copies on `stream` (cudaMemcpy2DAsync with cudaMemcpyDefault), so the
+ * sources may be device memory or pinned host memory.
+ *   k_rows, v_rows  bf16 [batch, h_kv, n_rows, d], dense;
+ *   k_cache, v_cache bf16 [batch, h_kv, t_cap, d].
+ * Constraints: 1 <= n_rows, t_ctx + n_rows <= t_cap.  No workspace.
+ */
+int bd_write_block_rows(const bd_shape* shape, int n_rows, const void* k_rows, const void* v_rows, void* k_cache,
+                        void* v_cache, void* stream);
 
 /*
  * Reads (and clears) the device status word of a workspace: BD_OK, or the first

@@ -2,8 +2,9 @@
 
 The hot path (KV-budget selection, gamma drafter decode passes over the sparse view, the
 verifier's causal block pass, the log-sum-exp merge and the greedy acceptance) lives in
-libbudgetdraft.so (hand-written CUDA, C ABI in include/budgetdraft.h).  This package holds its build step,
-a thin ctypes binding, a step runner and the seeded synthetic workloads.
+libbudgetdraft.so (hand-written CUDA, C ABI in include/budgetdraft.h).  This package holds
+its build step, a thin ctypes binding, a step runner, a pipelined host-buffer driver and the
+seeded synthetic workloads.
 """
 
 from .binding import (  # noqa: F401
@@ -27,9 +28,11 @@ from .binding import (  # noqa: F401
     bd_verify_attn,
     bd_workspace_size,
     bd_workspace_status,
+    bd_write_block_rows,
     library,
     make_shape,
     shape_of,
 )
 from .build import LIB_PATH, build  # noqa: F401
+from .hostio import HostStepIO  # noqa: F401
 from .step import SpecStep  # noqa: F401

@@ -52,6 +52,7 @@ _SIGNATURES = {
     "bd_accept": (ctypes.c_int, [ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P]),
     "bd_advance": (ctypes.c_int, [_SHAPE, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int, _P,
                                   _P]),
+    "bd_write_block_rows": (ctypes.c_int, [_SHAPE, ctypes.c_int, _P, _P, _P, _P, _P]),
     "bd_workspace_status": (ctypes.c_int, [_P, _P]),
     "bd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
 }
@@ -208,6 +209,14 @@ def bd_advance(shape, window, n_q, n_accept, q_verify, verify_lse, q_window, win
                               _ptr(verify_lse), _ptr(q_window), _ptr(window_lse), _ptr(idx), _ptr(count), cap,
                               _ptr(advance_out), _stream(stream))
     _check("bd_advance", st)
+
+
+def bd_write_block_rows(shape, n_rows, k_rows, v_rows, k_cache, v_cache, stream=None):
+    """Writes rows t_ctx .. t_ctx + n_rows - 1 of the caches from dense [b, h_kv, n_rows, d]
+    buffers (device or pinned host memory)."""
+    st = library().bd_write_block_rows(ctypes.byref(shape), int(n_rows), _ptr(k_rows), _ptr(v_rows), _ptr(k_cache),
+                                       _ptr(v_cache), _stream(stream))
+    _check("bd_write_block_rows", st)
 
 
 def bd_workspace_status(ws: Workspace, stream=None) -> int:

@@ -332,6 +332,29 @@ int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_acce
                                  idx_capacity, advance_out, static_cast<cudaStream_t>(stream)));
 }
 
+int bd_write_block_rows(const bd_shape* shape, int n_rows, const void* k_rows, const void* v_rows, void* k_cache,
+                        void* v_cache, void* stream) {
+  BD_TRY(check_shape(shape));
+  const bd_shape& s = *shape;
+  if (n_rows < 1 || s.t_ctx + n_rows > s.t_cap) return BD_ERR_INVALID_ARG;
+  BD_TRY(check_tensor(k_rows, 16));
+  BD_TRY(check_tensor(v_rows, 16));
+  BD_TRY(check_tensor(k_cache, 16));
+  BD_TRY(check_tensor(v_cache, 16));
+  const size_t row = (size_t)s.head_dim * 2;
+  const size_t units = (size_t)s.batch * s.h_kv;
+  const size_t width = (size_t)n_rows * row;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const void* src[2] = {k_rows, v_rows};
+  void* dst[2] = {k_cache, v_cache};
+  for (int i = 0; i < 2; ++i) {
+    uint8_t* d = static_cast<uint8_t*>(dst[i]) + (size_t)s.t_ctx * row;
+    if (cudaMemcpy2DAsync(d, (size_t)s.t_cap * row, src[i], width, width, units, cudaMemcpyDefault, st) != cudaSuccess)
+      return BD_ERR_CUDA;
+  }
+  return BD_OK;
+}
+
 int bd_workspace_status(void* ws, void* stream) {
   if (!ws) return BD_ERR_INVALID_ARG;
   int host = 0;

@@ -28,6 +28,13 @@ class SpecStep:
         self.verify_o = torch.empty(batch, h_q, gamma + 1, head_dim, dtype=torch.bfloat16, device=dev)
         self.verify_lse = torch.empty(batch, h_q, gamma + 1, dtype=torch.float32, device=dev)
 
+    def bind_outputs(self, idx, count, draft_o, draft_lse, verify_o, verify_lse):
+        """Directs the following calls' results into these tensors (same shapes and dtypes as
+        the ones allocated here)."""
+        self.idx, self.count = idx, count
+        self.draft_o, self.draft_lse = draft_o, draft_lse
+        self.verify_o, self.verify_lse = verify_o, verify_lse
+
     @classmethod
     def for_workload(cls, wl, budget=None, n_recent=None, chunk=1, device="cuda"):
         b = wl.budget if budget is None else budget

@@ -163,3 +163,12 @@ def test_advance_validation(lib):
     assert adv(shape(), qw=A + 8) == MISALIGNED
     assert adv(shape(), out=A + 2) == MISALIGNED
     assert adv(shape(head_dim=96)) == UNSUPPORTED
+
+
+def test_write_block_rows_validation(lib):
+    f = lib.bd_write_block_rows
+    assert f(ctypes.byref(shape()), 0, A, A, A, A, None) == INVALID
+    assert f(ctypes.byref(shape()), 11, A, A, A, A, None) == INVALID      # t_ctx + n_rows > t_cap
+    assert f(ctypes.byref(shape()), 6, A + 8, A, A, A, None) == MISALIGNED
+    assert f(ctypes.byref(shape()), 6, A, A, None, A, None) == INVALID
+    assert f(ctypes.byref(shape(head_dim=96)), 6, A, A, A, A, None) == UNSUPPORTED
