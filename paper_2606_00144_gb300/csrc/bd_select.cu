@@ -863,6 +863,260 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_token_kernel(const TopkP
   if (tid == 0) p.count_out[unit] = count;
 }
 
+// Token-level selection with every score held in registers (up to 16 per thread): the same
+// boundary-bin method as topk_token_kernel with the passes unrolled at compile time over
+// the thread's ROWS items, so no pass goes through shared memory but the histogram.  Warp w
+// owns items [w*ROWS*32, (w+1)*ROWS*32), row r of it at w*ROWS*32 + 32r + lane.  Needs
+// 0 < k < n <= ROWS * kTopkThreads.
+template <int ROWS>
+__global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkParams p) {
+  __shared__ uint32_t bins[kBins];
+  __shared__ uint64_t cand[kBinCandMax];
+  __shared__ uint32_t wsum[32];
+  __shared__ float wmin[32], wmax[32];
+  __shared__ uint32_t s_total, s_bin, s_above, s_nc, s_taukey, s_eq_take, s_eq_all, s_prefix, s_krem;
+  grid_dependency_wait();
+  allow_dependent_launch();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int unit = blockIdx.x;
+  const int lo = p.n_sink, hi = p.t_ctx - p.n_recent, n = hi - lo;
+  const int k = p.budget - p.n_sink - p.n_recent;
+  const float* sc = p.score + (size_t)unit * p.n_mid_pad;
+  int32_t* out = p.idx_out + (size_t)unit * p.budget;
+  const int w0 = warp * ROWS * 32;
+
+  // ---- the thread's scores (fp32 bits; non-negative, so their order is the bits' order)
+  uint32_t u[ROWS];
+  float lmin = INFINITY, lmax = -INFINITY;
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    const int i = w0 + 32 * r + lane;
+    const float v = i < n ? __ldcg(sc + i) : 0.f;
+    u[r] = __float_as_uint(v);
+    if (i < n) {
+      lmin = fminf(lmin, v);
+      lmax = fmaxf(lmax, v);
+    }
+  }
+  for (int i = tid; i < kBins; i += kTopkThreads) bins[i] = 0;
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, off));
+    lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, off));
+  }
+  if (lane == 0) {
+    wmin[warp] = lmin;
+    wmax[warp] = lmax;
+  }
+  if (tid == 0) {
+    s_nc = 0;
+    s_eq_take = 0;
+    s_eq_all = 0;
+  }
+  __syncthreads();
+  float vmin = wmin[0], vmax = wmax[0];
+#pragma unroll 8
+  for (int w = 1; w < 32; ++w) {
+    vmin = fminf(vmin, wmin[w]);
+    vmax = fmaxf(vmax, wmax[w]);
+  }
+
+  // ---- tau (bits of the k-th largest score) and krem (how many scores equal to tau to keep)
+  uint32_t tau = 0, krem = (uint32_t)k;
+  bool simple = false, found = false;
+  if (vmax > vmin) {
+    const float scale = (float)(kBins - 1) / (vmax - vmin);
+    auto bin_of = [&](uint32_t x) -> int { return min(kBins - 1, (int)((__uint_as_float(x) - vmin) * scale)); };
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r)
+      if (w0 + 32 * r + lane < n) atomicAdd(&bins[bin_of(u[r])], 1u);
+    __syncthreads();
+    constexpr int BPT = kBins / kTopkThreads;
+    uint32_t hb[BPT];
+    const uint4 hv = reinterpret_cast<const uint4*>(bins)[tid];
+    hb[0] = hv.x;
+    hb[1] = hv.y;
+    hb[2] = hv.z;
+    hb[3] = hv.w;
+    uint32_t incl = hb[0] + hb[1] + hb[2] + hb[3];
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t z = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += z;
+    }
+    if (lane == 31) wsum[warp] = incl;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t w = wsum[lane];
+      uint32_t c = w;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+        if (lane >= off) c += z;
+      }
+      wsum[lane] = c - w;
+      if (lane == 31) s_total = c;
+    }
+    __syncthreads();
+    uint32_t above = s_total - (wsum[warp] + incl);
+#pragma unroll
+    for (int j = BPT - 1; j >= 0; --j) {
+      if (above < (uint32_t)k && (uint32_t)k <= above + hb[j]) {
+        s_bin = (uint32_t)(tid * BPT + j);
+        s_above = above;
+        s_prefix = hb[j];
+      }
+      above += hb[j];
+    }
+    __syncthreads();
+    const int bstar = (int)s_bin;
+    const uint32_t nc = s_prefix;
+    if (nc <= (uint32_t)kBinCandMax) {
+#pragma unroll
+      for (int r = 0; r < ROWS; ++r) {
+        const int i = w0 + 32 * r + lane;
+        if (i < n && bin_of(u[r]) == bstar)
+          cand[atomicAdd(&s_nc, 1u)] = (static_cast<uint64_t>(u[r]) << 32) | (0xFFFFFFFFu - (uint32_t)i);
+      }
+      __syncthreads();
+      const uint32_t m = (uint32_t)k - s_above;
+      for (int i = tid; i < (int)nc; i += kTopkThreads) {
+        const uint64_t kk = cand[i];
+        uint32_t rk = 0;
+        for (int j = 0; j < (int)nc; ++j) rk += cand[j] > kk;
+        if (rk == m - 1) s_taukey = static_cast<uint32_t>(kk >> 32);
+      }
+      __syncthreads();
+      tau = s_taukey;
+      for (int i = tid; i < (int)nc; i += kTopkThreads) {
+        const uint64_t kk = cand[i];
+        if (static_cast<uint32_t>(kk >> 32) != tau) continue;
+        uint32_t rk = 0;
+        for (int j = 0; j < (int)nc; ++j) rk += cand[j] > kk;
+        atomicAdd(&s_eq_all, 1u);
+        if (rk < m) atomicAdd(&s_eq_take, 1u);
+      }
+      __syncthreads();
+      krem = s_eq_take;
+      simple = (s_eq_take == s_eq_all);
+      found = true;
+    }
+  }
+  if (!found) {
+    // crowded boundary (many equal or near-equal scores): exact 4-pass radix select
+    uint32_t prefix = 0, mask = 0;
+    krem = (uint32_t)k;
+    for (int pass = 0; pass < 4; ++pass) {
+      const int shift = 24 - 8 * pass;
+      for (int i = tid; i < 256; i += kTopkThreads) bins[i] = 0;
+      __syncthreads();
+#pragma unroll
+      for (int r = 0; r < ROWS; ++r)
+        if (w0 + 32 * r + lane < n && (u[r] & mask) == prefix) atomicAdd(&bins[(u[r] >> shift) & 255u], 1u);
+      __syncthreads();
+      if (warp == 0) {
+        uint32_t local = 0;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) local += bins[8 * lane + j];
+        uint32_t suffix = local;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const uint32_t y = __shfl_down_sync(0xffffffffu, suffix, off);
+          if (lane + off < 32) suffix += y;
+        }
+        uint32_t abv = suffix - local;
+        if (abv < krem && krem <= suffix) {
+          for (int j = 7; j >= 0; --j) {
+            const uint32_t h = bins[8 * lane + j];
+            if (abv + h >= krem) {
+              s_prefix = prefix | ((uint32_t)(8 * lane + j) << shift);
+              s_krem = krem - abv;
+              break;
+            }
+            abv += h;
+          }
+        }
+      }
+      __syncthreads();
+      prefix = s_prefix;
+      krem = s_krem;
+      mask |= 0xFFu << shift;
+    }
+    tau = prefix;
+    simple = false;
+  }
+
+  // ---- ascending compaction: warp ballots of the selected items, block scan, writes
+  const uint32_t lt = (1u << lane) - 1u;
+  uint32_t eq_base = 0;
+  if (!simple) {
+    // items equal to tau are taken in position order: count those before this warp's items
+    uint32_t eqc = 0;
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r)
+      eqc += __popc(__ballot_sync(0xffffffffu, w0 + 32 * r + lane < n && u[r] == tau));
+    if (lane == 0) wsum[warp] = eqc;
+    __syncthreads();
+    if (warp == 0) {
+      const uint32_t w = wsum[lane];
+      uint32_t c = w;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+        if (lane >= off) c += z;
+      }
+      wsum[lane] = c - w;
+    }
+    __syncthreads();
+    eq_base = wsum[warp];
+    __syncthreads();
+  }
+  uint32_t masks[ROWS];
+  uint32_t cnt = 0, eq_run = eq_base;
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    const bool valid = w0 + 32 * r + lane < n;
+    bool sel = valid && u[r] > tau;
+    const bool eq = valid && u[r] == tau;
+    if (simple) {
+      sel |= eq;
+    } else {
+      const uint32_t be = __ballot_sync(0xffffffffu, eq);
+      if (eq) sel = eq_run + __popc(be & lt) < krem;
+      eq_run += __popc(be);
+    }
+    masks[r] = __ballot_sync(0xffffffffu, sel);
+    cnt += __popc(masks[r]);
+  }
+  if (lane == 0) wsum[warp] = cnt;
+  __syncthreads();
+  if (warp == 0) {
+    const uint32_t w = wsum[lane];
+    uint32_t c = w;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
+      if (lane >= off) c += z;
+    }
+    wsum[lane] = c - w;
+    if (lane == 31) s_total = c;
+  }
+  __syncthreads();
+  uint32_t base = (uint32_t)lo + wsum[warp];
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    const uint32_t mk = masks[r];
+    if ((mk >> lane) & 1u) out[base + __popc(mk & lt)] = lo + w0 + 32 * r + lane;
+    base += __popc(mk);
+  }
+  const int n_chosen = (int)s_total;
+  const int count = lo + n_chosen + p.n_recent;
+  for (int i = tid; i < lo; i += kTopkThreads) out[i] = i;
+  for (int i = tid; i < p.n_recent; i += kTopkThreads) out[lo + n_chosen + i] = hi + i;
+  for (int i = count + tid; i < p.budget; i += kTopkThreads) out[i] = -1;
+  if (tid == 0) p.count_out[unit] = count;
+}
+
 // ============================================================================ host side
 
 namespace {
@@ -999,6 +1253,15 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
   tp.keep_all = plan.keep_all ? 1 : 0;
   void* targs[] = {&tp};
   const int free = budget - n_sink - n_recent;
+  if (!plan.keep_all && plan.need_scores && chunk == 1 && free < plan.n_mid && plan.n_mid <= 16 * kTopkThreads) {
+    const int rows = (plan.n_mid + kTopkThreads - 1) / kTopkThreads;
+    void* fn = rows <= 1   ? reinterpret_cast<void*>(&topk_rows_kernel<1>)
+               : rows <= 2 ? reinterpret_cast<void*>(&topk_rows_kernel<2>)
+               : rows <= 4 ? reinterpret_cast<void*>(&topk_rows_kernel<4>)
+               : rows <= 8 ? reinterpret_cast<void*>(&topk_rows_kernel<8>)
+                           : reinterpret_cast<void*>(&topk_rows_kernel<16>);
+    return launch_kernel(fn, dim3(units), dim3(kTopkThreads), 0, stream, targs, 0);
+  }
   if (!plan.keep_all && plan.need_scores && chunk == 1 && plan.n_mid <= kLeanMaxItems && free < plan.n_mid) {
     const size_t smem = (size_t)align_up(plan.n_mid, 4) * 4;
     void* fn = reinterpret_cast<void*>(&topk_token_kernel);

@@ -197,6 +197,8 @@ RAGGED = [
     (1, 8, 2, 128, 1031, 128, 4, 32, 32, 5, 8),   # chunks with sink/recent and ragged chunk edges
     (1, 8, 2, 128, 300, 36, 4, 32, 32, 1, 1),     # B = sink + recent: nothing ranked
     (1, 8, 2, 64, 40, 64, 4, 8, 32, 5, 1),        # B > T
+    (1, 8, 2, 128, 20000, 600, 4, 64, 32, 1, 1),  # 16K < middle <= 32K: the shared-memory top-B kernel
+    (1, 4, 1, 64, 40000, 300, 4, 32, 32, 1, 1),   # middle > 32K: the general top-B kernel
 ]
 
 
