@@ -110,3 +110,57 @@ def test_multistep_carry_selection_on_the_slid_window():
         err = np.abs(lse_win.cpu().double().numpy() - oracle.window_lse(qh[:, :, t - W: t], Kh, t)).max()
         assert err <= 1e-3, f"step {step}: slid window LSE off by {err}"
         assert ws.status() == 0
+
+
+def test_amortised_loop_view_grows_by_the_settled_rows():
+    """Algorithm 2 as written: sparsify once, then every step appends its settled rows to the
+    drafter's view.  After each advance the next step's draft pass must equal the oracle's
+    draft attention over (first selection + every appended position)."""
+    b, hq, hkv, d, W, gamma = 2, 8, 2, 128, 32, 3
+    t0, steps, budget, sink, recent = 2000, 3, 128, 4, 32
+    cap_rows = t0 + steps * (gamma + 1)
+    capacity = budget + steps * (gamma + 1)
+    g = torch.Generator().manual_seed(91)
+    K, V = bf16_randn(g, b, hkv, cap_rows, d).cuda(), bf16_randn(g, b, hkv, cap_rows, d).cuda()
+    q_all = bf16_randn(g, b, hq, cap_rows, d).cuda()
+    qd_all = bf16_randn(g, steps, gamma, b, hq, d).cuda()          # drafter queries of every pass
+    Kh, Vh = f64(K), f64(V)
+    rng = np.random.default_rng(8)
+    t = t0
+    shape = bd.make_shape(b, hq, hkv, d, t, cap_rows)
+    idx = torch.full((b, hkv, capacity), -1, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(b, hkv, dtype=torch.int32, device="cuda")
+    ws = bd.Workspace.for_step(shape, budget, W, gamma)
+    q_win = q_all[:, :, t - W: t].contiguous()
+    sel = torch.full((b, hkv, budget), -1, dtype=torch.int32, device="cuda")
+    bd.bd_select_budget(shape, K, q_win, None, W, budget, sink, recent, 1, sel, cnt, ws)
+    idx[:, :, :budget] = sel
+    lse_win = torch.empty(b, hq, W, dtype=torch.float32, device="cuda")
+    vo = torch.empty(b, hq, gamma + 1, d, dtype=torch.bfloat16, device="cuda")
+    vl = torch.empty(b, hq, gamma + 1, dtype=torch.float32, device="cuda")
+    do = torch.empty(b, hq, d, dtype=torch.bfloat16, device="cuda")
+    dl = torch.empty(b, hq, dtype=torch.float32, device="cuda")
+    adv = torch.zeros(1, dtype=torch.int32, device="cuda")
+    for step in range(steps):
+        shape = bd.make_shape(b, hq, hkv, d, t, cap_rows)
+        ws = bd.Workspace.for_step(shape, capacity, W, gamma)
+        torch.cuda.synchronize()
+        idx_h, cnt_h = idx.cpu().numpy(), cnt.cpu().numpy()
+        for j in range(gamma):
+            q = qd_all[step, j].contiguous()
+            bd.bd_draft_attn(shape, q, K, V, idx, cnt, capacity, j, do, dl, ws)
+            o_ref, l_ref = oracle.draft_attn(f64(q), Kh, Vh, idx_h, cnt_h, t, j)
+            torch.cuda.synchronize()
+            check_attention(do, dl, o_ref, l_ref, f"step {step} draft {j}")
+        q_ver = q_all[:, :, t: t + gamma + 1].contiguous()
+        bd.bd_verify_attn(shape, q_ver, gamma + 1, K, V, vo, vl, ws)
+        n_acc = rng.integers(0, gamma + 1, size=b)
+        bd.bd_advance(shape, W, gamma + 1, torch.from_numpy(n_acc).int().cuda(), q_ver, vl, q_win, lse_win, idx,
+                      cnt, adv)
+        torch.cuda.synchronize()
+        a = int(adv.item())
+        i_ref, c_ref, full = oracle.append_view(idx_h, cnt_h, t, a, capacity)
+        assert not full
+        assert idx.cpu().numpy().tolist() == i_ref.tolist() and cnt.cpu().numpy().tolist() == c_ref.tolist()
+        t += a
+        assert ws.status() == 0
