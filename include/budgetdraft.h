@@ -2,7 +2,8 @@
  * budgetdraft.h - C ABI of the speculative-step attention library (libbudgetdraft.so).
  *
  * One speculative step of BudgetDraft (arXiv 2606.00144, Algorithm 2) spends its
- * KV-cache attention in three places, each an entry point below:
+ * KV-cache attention in three places, each an entry point below, plus the merge they
+ * share:
  *   bd_select_budget  builds the drafter's sparse view K_S^sp(B) under a KV budget B
  *                     (Sec. 3.4 TopKChunks; Algorithm 2, sparsify);
  *   bd_draft_attn     one of the gamma drafter decode passes over that view
@@ -21,8 +22,9 @@
  *                     appends their positions to the sparse view (Algorithm 2, Update).
  *
  * Conventions shared by every call
- *   - All tensor arguments are DEVICE pointers owned by the caller; the library
- *     never allocates, frees or keeps a pointer after a call returns.
+ *   - All tensor arguments are DEVICE pointers owned by the caller (the row sources
+ *     of bd_write_block_rows may also be pinned host memory); the library never
+ *     allocates, frees or keeps a pointer after a call returns.
  *   - bf16 tensors are IEEE bfloat16 (raw 16-bit), fp32 are IEEE float, int32 are
  *     int32_t.  Every tensor is dense row-major in the order written.  bf16 tensors
  *     (caches, queries, outputs) and fp32 split-K partials must be 16-byte aligned;
