@@ -9,9 +9,11 @@
 //                          unit's window queries into a double-buffered swizzled Q tile;
 //                          both are context data, streamed before the grid-dependency
 //                          wait, which only the epilogue (reading the window LSE) takes;
-//                 warp 1   one lane issues tcgen05.mma into a double-buffered fp32 TMEM
-//                          accumulator and commits to the smem/TMEM barriers;
-//                 warps 2-5 epilogue: tcgen05.ld, ex2 (MUFU), row sums, coalesced store.
+//                 warp 1   one lane issues tcgen05.mma into four fp32 TMEM accumulators
+//                          (two when the window rows need more columns) and commits to
+//                          the smem/TMEM barriers;
+//                 warps 2-9 epilogue (two groups of 4, alternate tiles): tcgen05.ld,
+//                          packed f32x2 FMA, ex2 (MUFU), packed row sums, coalesced store.
 // topk_kernel   one CTA per (sequence, KV head), scores staged in shared memory: a linear
 //               histogram between the min and max score finds the bin holding the k-th
 //               largest; that bin's few items are ranked exactly by (score desc, position
@@ -189,7 +191,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     const int grp = (warp - 2) >> 2;            // group 0: warps 2-5, group 1: warps 6-9; tiles i % 2 == grp
     const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
     const int ep_tid = (warp - 2 - 4 * grp) * 32 + lane;
-    float* lse2_s = reinterpret_cast<float*>(smem + 1024 + grp * 2304);   // [288]
+    float* lse2_s = reinterpret_cast<float*>(smem + 1024 + grp * 2304);   // [288] -lse * log2(e)
     int* pw_s = reinterpret_cast<int*>(smem + 1024 + grp * 2304 + 1152);  // [288]
     const int win0 = p.t_ctx - p.window;        // position of window row 0
     int cur_unit = -1;
@@ -200,7 +202,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
         named_bar(1 + grp, 128);
         for (int c = ep_tid; c < 288; c += 128) {
           const bool real = c < p.nq_rows;
-          lse2_s[c] = real ? __ldg(p.lse_win + (size_t)unit * p.nq_rows + c) * kLog2e : INFINITY;
+          lse2_s[c] = real ? -__ldg(p.lse_win + (size_t)unit * p.nq_rows + c) * kLog2e : -INFINITY;
           pw_s[c] = real ? win0 + c % p.window : -1;
         }
         named_bar(1 + grp, 128);
@@ -221,18 +223,32 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
         tc_wait_ld();
         const int ncol = min(64, p.nq_pad - c0);
         if (ncol == 64 && !causal) {
+          // packed pairs: one f32x2 FMA and one f32x2 add per two scores (the epilogue's
+          // instruction issue, not the exponentials, limits this loop)
+          const float2 cc = make_float2(p.scale_log2, p.scale_log2);
+          float2 a0 = make_float2(0.f, 0.f), a1 = a0, a2 = a0, a3 = a0;
 #pragma unroll
-          for (int j = 0; j < 64; j += 4) {
-            sum0 += fast_exp2(fmaf(v[j], p.scale_log2, -lse2_s[c0 + j]));
-            sum1 += fast_exp2(fmaf(v[j + 1], p.scale_log2, -lse2_s[c0 + j + 1]));
-            sum2 += fast_exp2(fmaf(v[j + 2], p.scale_log2, -lse2_s[c0 + j + 2]));
-            sum3 += fast_exp2(fmaf(v[j + 3], p.scale_log2, -lse2_s[c0 + j + 3]));
+          for (int j = 0; j < 64; j += 8) {
+            const float4 la = *reinterpret_cast<const float4*>(lse2_s + c0 + j);
+            const float4 lb = *reinterpret_cast<const float4*>(lse2_s + c0 + j + 4);
+            const float2 x0 = ffma2(make_float2(v[j], v[j + 1]), cc, make_float2(la.x, la.y));
+            const float2 x1 = ffma2(make_float2(v[j + 2], v[j + 3]), cc, make_float2(la.z, la.w));
+            const float2 x2 = ffma2(make_float2(v[j + 4], v[j + 5]), cc, make_float2(lb.x, lb.y));
+            const float2 x3 = ffma2(make_float2(v[j + 6], v[j + 7]), cc, make_float2(lb.z, lb.w));
+            a0 = fadd2(a0, make_float2(fast_exp2(x0.x), fast_exp2(x0.y)));
+            a1 = fadd2(a1, make_float2(fast_exp2(x1.x), fast_exp2(x1.y)));
+            a2 = fadd2(a2, make_float2(fast_exp2(x2.x), fast_exp2(x2.y)));
+            a3 = fadd2(a3, make_float2(fast_exp2(x3.x), fast_exp2(x3.y)));
           }
+          sum0 += a0.x + a0.y;
+          sum1 += a1.x + a1.y;
+          sum2 += a2.x + a2.y;
+          sum3 += a3.x + a3.y;
         } else {
 #pragma unroll
           for (int j = 0; j < 64; ++j) {
             if (j < ncol) {
-              const float x = key <= pw_s[c0 + j] ? fmaf(v[j], p.scale_log2, -lse2_s[c0 + j]) : -INFINITY;
+              const float x = key <= pw_s[c0 + j] ? fmaf(v[j], p.scale_log2, lse2_s[c0 + j]) : -INFINITY;
               sum0 += fast_exp2(x);
             }
           }
