@@ -68,7 +68,13 @@ typedef enum bd_status {
   BD_ERR_TIMEOUT = -6       /* device side: a bounded wait ran out (status word only)    */
 } bd_status;
 
-/* Problem shape of one layer's cache.  The caches are [batch, h_kv, t_cap, head_dim]. */
+/* Problem shape of one layer's cache.  The caches are [batch, h_kv, t_cap, head_dim].
+ * seq_lens (optional) gives every sequence its own context length T_b: a DEVICE int32
+ * array [batch] with 1 <= T_b <= t_ctx, read by the kernels (so a step's lengths can be
+ * advanced on the device by bd_advance); t_ctx is then the longest length and sizes the
+ * launches.  Everything this header says of t_ctx holds per sequence with T_b in its
+ * place.  NULL: every sequence has t_ctx.  A T_b outside [1, t_ctx] is recorded in the
+ * workspace status word (BD_ERR_INVALID_ARG) and clamped into range. */
 typedef struct bd_shape {
   int32_t batch;     /* sequences                                   */
   int32_t h_q;       /* query heads                                 */
@@ -76,6 +82,7 @@ typedef struct bd_shape {
   int32_t head_dim;  /* d: 64 or 128                                 */
   int32_t t_ctx;     /* context length T (cached prefix positions)   */
   int32_t t_cap;     /* rows per (sequence, KV head) in the arrays   */
+  const int32_t* seq_lens;  /* per-sequence lengths [batch] or NULL  */
 } bd_shape;
 
 /* Element types of bd_argmax logits. */
@@ -237,12 +244,14 @@ int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* 
 /*
  * Cache update after acceptance (Algorithm 2, Update).  The verify block held positions
  * t_ctx .. t_ctx + n_q - 1 (the token the step started from, then the drafts); after
- * acceptance of k_b drafts, sequence b's rows t_ctx .. t_ctx + k_b are settled.  One call
- * shares one context length over the batch, so the batch advances by
- *     a = min_b(clamp(n_accept[b], 0, n_q - 1)) + 1
- * positions (every sequence stays on tokens its verifier confirmed).  The K/V rows of the
- * block were written into the caches before bd_verify_attn and stay where they are: the
- * caller makes the settled ones context by using t_ctx + a as the next step's t_ctx.
+ * acceptance of k_b drafts, sequence b's rows t_ctx .. t_ctx + k_b are settled, a_b =
+ * clamp(n_accept[b], 0, n_q - 1) + 1 rows.  The K/V rows of the block were written into
+ * the caches before bd_verify_attn and stay where they are.
+ *   - Per-sequence lengths (shape->seq_lens set): sequence b advances by its own a_b, and
+ *     this call adds a_b to seq_lens[b] on the device (the array is updated in place).
+ *   - One shared length (seq_lens NULL): the batch advances by a = min_b a_b (every
+ *     sequence stays on tokens its verifier confirmed); the caller uses t_ctx + a as the
+ *     next step's t_ctx.
  * This call updates the state that carry-mode selection and the drafter need:
  *   - q_window / window_lse slide by a: they hold positions t_ctx + a - W ..
  *     t_ctx + a - 1 afterwards, the new rows taken from q_verify / verify_lse (the
@@ -250,6 +259,7 @@ int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* 
  *   - idx / count (optional): positions t_ctx .. t_ctx + a - 1 are appended to every
  *     unit's view (Algorithm 2 appends accepted tokens to the sparse cache); a unit
  *     whose view has no room (count + a > idx_capacity) is left unchanged.
+ * (with per-sequence lengths, read T_b for t_ctx and a_b for a in both items.)
  *   n_accept      int32 [batch] accepted drafts per sequence (bd_accept's n_accept_out);
  *   q_verify      bf16 [batch, h_q, n_q, d]; verify_lse fp32 [batch, h_q, n_q] (NULL
  *                 together with window_lse);
@@ -257,7 +267,7 @@ int bd_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* 
  *                 read and rewritten in place;
  *   idx           int32 [batch, h_kv, idx_capacity], count int32 [batch, h_kv] (both
  *                 NULL to skip the view);
- *   advance_out   int32 [1]: a (may be NULL).
+ *   advance_out   int32 [batch]: each sequence's advance (may be NULL).
  * Constraints: 1 <= window <= t_ctx, 1 <= n_q, t_ctx + n_q <= t_cap.  No workspace.
  */
 int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_accept, const void* q_verify,
@@ -267,8 +277,9 @@ int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_acce
 /*
  * Writes the K/V rows of the current block into the caches: rows t_ctx .. t_ctx + n_rows - 1
  * of every (sequence, KV head) (Algorithm 2, Update: new tokens' keys and values join the
- * cache).  Two strided copies on `stream` (cudaMemcpy2DAsync with cudaMemcpyDefault), so the
- * sources may be device memory or pinned host memory.
+ * cache).  Two strided copies on `stream` (cudaMemcpy2DAsync with cudaMemcpyDefault), or with
+ * per-sequence lengths one kernel that writes rows T_b .. T_b + n_rows - 1; the sources may
+ * be device memory or pinned host memory either way.
  *   k_rows, v_rows  bf16 [batch, h_kv, n_rows, d], dense;
  *   k_cache, v_cache bf16 [batch, h_kv, t_cap, d].
  * Constraints: 1 <= n_rows, t_ctx + n_rows <= t_cap.  No workspace.

@@ -22,7 +22,8 @@ BD_DTYPE_BF16, BD_DTYPE_F32 = 1, 2
 
 class BdShape(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int32), ("h_q", ctypes.c_int32), ("h_kv", ctypes.c_int32),
-                ("head_dim", ctypes.c_int32), ("t_ctx", ctypes.c_int32), ("t_cap", ctypes.c_int32)]
+                ("head_dim", ctypes.c_int32), ("t_ctx", ctypes.c_int32), ("t_cap", ctypes.c_int32),
+                ("seq_lens", ctypes.c_void_p)]
 
     def __repr__(self):
         return (f"BdShape(batch={self.batch}, h_q={self.h_q}, h_kv={self.h_kv}, head_dim={self.head_dim}, "
@@ -102,8 +103,10 @@ def _check(name, status):
         raise BudgetDraftError(name, status)
 
 
-def make_shape(batch, h_q, h_kv, head_dim, t_ctx, t_cap) -> BdShape:
-    return BdShape(int(batch), int(h_q), int(h_kv), int(head_dim), int(t_ctx), int(t_cap))
+def make_shape(batch, h_q, h_kv, head_dim, t_ctx, t_cap, seq_lens=None) -> BdShape:
+    """seq_lens: optional int32 device tensor [batch] of per-sequence context lengths (t_ctx
+    is then the longest); the tensor must outlive every call made with this shape."""
+    return BdShape(int(batch), int(h_q), int(h_kv), int(head_dim), int(t_ctx), int(t_cap), _ptr(seq_lens))
 
 
 def shape_of(k_cache: torch.Tensor, h_q: int, t_ctx: int) -> BdShape:

@@ -225,14 +225,18 @@ struct AdvanceParams {
   float* lse_win;                 // [batch, h_q, window] or null
   int32_t* idx;                   // [batch, h_kv, capacity] or null
   int32_t* count;                 // [batch, h_kv]
-  int32_t* advance_out;           // [1] or null
+  int32_t* advance_out;           // [batch] or null
+  int32_t* seq_lens;              // per-sequence context lengths [batch], advanced in place, or null
   int batch, h_q, h_kv, window, n_q, t_ctx, capacity;
 };
 
 // grid (h_q, batch).  CTA (h, b) slides the window of query head h of sequence b: new row w
 // is old row w + a while that exists, else block row w + a - window.  The new rows are
-// staged in shared memory before any is written, so the slide is done in place.  CTAs with
-// h < h_kv also append the positions t_ctx .. t_ctx + a - 1 to the view of unit (b, h).
+// staged in shared memory before any is written, so the slide is done in place.  With one
+// shared length, a is the batch minimum of the settled counts and CTAs with h < h_kv append
+// positions t_ctx .. t_ctx + a - 1 to the view of unit (b, h); with per-sequence lengths,
+// a is sequence b's own count and CTA (0, b) appends T_b .. T_b + a - 1 to all of the
+// sequence's views, then advances T_b (no other CTA reads it).
 template <int D>
 __global__ void __launch_bounds__(kVThreads) advance_kernel(const AdvanceParams p) {
   extern __shared__ __align__(16) uint8_t adv_smem[];
@@ -240,17 +244,22 @@ __global__ void __launch_bounds__(kVThreads) advance_kernel(const AdvanceParams 
   grid_dependency_wait();
   allow_dependent_launch();
   const int tid = threadIdx.x, h = blockIdx.x, b = blockIdx.y;
-  int m = INT_MAX;
-  for (int i = tid; i < p.batch; i += kVThreads) m = min(m, p.n_accept[i]);
+  int m;
+  if (p.seq_lens) {
+    m = p.n_accept[b];
+  } else {
+    m = INT_MAX;
+    for (int i = tid; i < p.batch; i += kVThreads) m = min(m, p.n_accept[i]);
 #pragma unroll
-  for (int off = 16; off > 0; off >>= 1) m = min(m, __shfl_xor_sync(0xffffffffu, m, off));
-  if ((tid & 31) == 0) s_min[tid >> 5] = m;
-  __syncthreads();
-  m = s_min[0];
+    for (int off = 16; off > 0; off >>= 1) m = min(m, __shfl_xor_sync(0xffffffffu, m, off));
+    if ((tid & 31) == 0) s_min[tid >> 5] = m;
+    __syncthreads();
+    m = s_min[0];
 #pragma unroll
-  for (int w = 1; w < kVThreads / 32; ++w) m = min(m, s_min[w]);
+    for (int w = 1; w < kVThreads / 32; ++w) m = min(m, s_min[w]);
+  }
   const int a = min(max(m, 0), p.n_q - 1) + 1;       // settled rows: the start token + k accepted
-  if (h == 0 && b == 0 && tid == 0 && p.advance_out) p.advance_out[0] = a;
+  if (h == 0 && tid == 0 && p.advance_out) p.advance_out[b] = a;
 
   const int W = p.window;
   constexpr int CH = D / 8;                         // 16-byte chunks per row
@@ -275,15 +284,66 @@ __global__ void __launch_bounds__(kVThreads) advance_kernel(const AdvanceParams 
   if (p.lse_win)
     for (int w = tid; w < W; w += kVThreads) p.lse_win[bh * W + w] = ls[w];
 
-  if (p.idx && h < p.h_kv) {
-    const size_t u = (size_t)b * p.h_kv + h;
-    const int c = p.count[u];
-    if (c + a <= p.capacity) {                      // a view without room is left as it is
-      for (int i = tid; i < a; i += kVThreads) p.idx[u * p.capacity + c + i] = p.t_ctx + i;
-      __syncthreads();
-      if (tid == 0) p.count[u] = c + a;
+  if (p.seq_lens == nullptr) {
+    if (p.idx && h < p.h_kv) {
+      const size_t u = (size_t)b * p.h_kv + h;
+      const int c = p.count[u];
+      if (c + a <= p.capacity) {                    // a view without room is left as it is
+        for (int i = tid; i < a; i += kVThreads) p.idx[u * p.capacity + c + i] = p.t_ctx + i;
+        __syncthreads();
+        if (tid == 0) p.count[u] = c + a;
+      }
     }
+  } else if (h == 0) {
+    const int t_b = p.seq_lens[b];
+    if (p.idx) {
+      for (int g = 0; g < p.h_kv; ++g) {
+        const size_t u = (size_t)b * p.h_kv + g;
+        const int c = p.count[u];
+        if (c + a <= p.capacity) {
+          for (int i = tid; i < a; i += kVThreads) p.idx[u * p.capacity + c + i] = t_b + i;
+          __syncthreads();
+          if (tid == 0) p.count[u] = c + a;
+        }
+      }
+    }
+    __syncthreads();
+    if (tid == 0) p.seq_lens[b] = t_b + a;
   }
+}
+
+// grid (units): rows T_u .. T_u + n_rows - 1 of unit u's K and V rows from dense
+// [units][n_rows][D] sources (device or pinned host memory, read through the unified
+// address space), for per-sequence lengths.
+template <int D>
+__global__ void __launch_bounds__(128) write_rows_kernel(const uint4* k_rows, const uint4* v_rows, uint4* k_cache,
+                                                         uint4* v_cache, const int32_t* seq_lens, int h_kv,
+                                                         int t_cap, int n_rows) {
+  grid_dependency_wait();
+  allow_dependent_launch();
+  constexpr int CH = D / 8;
+  const int u = blockIdx.x;
+  const int t_u = seq_lens[u / h_kv];
+  const size_t src0 = (size_t)u * n_rows * CH;
+  const size_t dst0 = ((size_t)u * t_cap + t_u) * CH;
+  for (int i = threadIdx.x; i < n_rows * CH; i += blockDim.x) {
+    k_cache[dst0 + i] = k_rows[src0 + i];
+    v_cache[dst0 + i] = v_rows[src0 + i];
+  }
+}
+
+cudaError_t launch_write_rows(const bd_shape& s, int n_rows, const void* k_rows, const void* v_rows, void* k_cache,
+                              void* v_cache, cudaStream_t stream) {
+  const uint4* kr = static_cast<const uint4*>(k_rows);
+  const uint4* vr = static_cast<const uint4*>(v_rows);
+  uint4* kc = static_cast<uint4*>(k_cache);
+  uint4* vc = static_cast<uint4*>(v_cache);
+  const int32_t* lens = s.seq_lens;
+  int h_kv = s.h_kv, t_cap = s.t_cap;
+  void* args[] = {&kr, &vr, &kc, &vc, const_cast<int32_t**>(&lens), &h_kv, &t_cap, &n_rows};
+  void* fn = s.head_dim == 64 ? reinterpret_cast<void*>(&write_rows_kernel<64>)
+                              : reinterpret_cast<void*>(&write_rows_kernel<128>);
+  return launch_kernel(fn, dim3(s.batch * s.h_kv), dim3(128), 0, stream, args, 0);
 }
 
 size_t advance_smem(int window, int head_dim) { return (size_t)window * head_dim * 2 + (size_t)window * 4; }
@@ -300,6 +360,7 @@ cudaError_t launch_advance(const bd_shape& s, int window, int n_q, const int32_t
   p.idx = idx;
   p.count = count;
   p.advance_out = advance_out;
+  p.seq_lens = const_cast<int32_t*>(s.seq_lens);
   p.batch = s.batch;
   p.h_q = s.h_q;
   p.h_kv = s.h_kv;

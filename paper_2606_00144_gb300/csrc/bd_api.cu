@@ -104,6 +104,7 @@ int check_shape(const bd_shape* s) {
   if (s->head_dim != 64 && s->head_dim != 128) return BD_ERR_UNSUPPORTED;
   // every per-unit row offset must stay addressable by the TMA (rows < 2^31)
   if ((long long)s->batch * s->h_kv * s->t_cap >= (1LL << 31)) return BD_ERR_UNSUPPORTED;
+  if (s->seq_lens && !aligned(s->seq_lens, 4)) return BD_ERR_MISALIGNED;
   return BD_OK;
 }
 
@@ -341,10 +342,11 @@ int bd_write_block_rows(const bd_shape* shape, int n_rows, const void* k_rows, c
   BD_TRY(check_tensor(v_rows, 16));
   BD_TRY(check_tensor(k_cache, 16));
   BD_TRY(check_tensor(v_cache, 16));
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (s.seq_lens) return map_cuda(launch_write_rows(s, n_rows, k_rows, v_rows, k_cache, v_cache, st));
   const size_t row = (size_t)s.head_dim * 2;
   const size_t units = (size_t)s.batch * s.h_kv;
   const size_t width = (size_t)n_rows * row;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   const void* src[2] = {k_rows, v_rows};
   void* dst[2] = {k_cache, v_cache};
   for (int i = 0; i < 2; ++i) {

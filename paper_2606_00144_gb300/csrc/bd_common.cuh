@@ -285,6 +285,19 @@ __host__ __device__ constexpr uint32_t umma_idesc_bf16(int m, int n) {
          (static_cast<uint32_t>(m >> 4) << 24);
 }
 
+// Context length of the sequence that owns (sequence, KV head) unit `unit` (units are
+// sequence-major): seq_lens[unit / h_kv] when per-sequence lengths are given, else t_ctx.
+// A length outside [1, t_ctx] is recorded as an argument error and clamped.
+__device__ __forceinline__ int unit_context(const int32_t* seq_lens, int unit, int h_kv, int t_ctx, int* status) {
+  if (seq_lens == nullptr) return t_ctx;
+  int t = seq_lens[unit / h_kv];
+  if (t < 1 || t > t_ctx) {
+    if (status) record_error(status, BD_ERR_INVALID_ARG);
+    t = min(max(t, 1), t_ctx);
+  }
+  return t;
+}
+
 // ---------------------------------------------------------------------------------------
 // Log-sum-exp merge of split partials (shared by the fused split-K paths and bd_combine)
 // ---------------------------------------------------------------------------------------

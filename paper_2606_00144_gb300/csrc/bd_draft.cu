@@ -43,6 +43,8 @@ struct DraftParams {
   __nv_bfloat16* o;            // [units * G][D]
   float* lse;                  // [units * G] or null
   int* status;
+  const int32_t* seq_lens;      // per-sequence context lengths [batch] or null (all t_ctx)
+  int h_kv;
   int budget, step_j, t_ctx, t_cap, n_split, rows_per_split;
   int n_stage;                 // 1, or 2 when a CTA gathers more than one tile (double buffer)
   unsigned flags;              // BD_DRAFT_VIEW_READY: gather the selected rows before the dependency wait
@@ -103,6 +105,9 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     if (tid == 0) record_error(p.status, BD_ERR_INVALID_ARG);
     cnt = min(max(cnt, 0), p.budget);
   }
+  // the unit's context length (like idx and count, written before the preceding kernel
+  // when the view is ready, so it may be read before the dependency wait)
+  const int t_unit = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
   const int n_entries = cnt + p.step_j + 1;
   const int e_end = min(e_begin + p.rows_per_split, n_entries);
   const int n_tiles = e_end > e_begin ? (e_end - e_begin + kDRows - 1) / kDRows : 0;
@@ -110,8 +115,8 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   const __nv_bfloat16* vunit = p.v + (size_t)unit * p.t_cap * D;
 
   auto position = [&](int e, int idx_value) -> int {
-    if (e >= cnt) return p.t_ctx + (e - cnt);            // a drafted row
-    if (idx_value < 0 || idx_value >= p.t_ctx) {
+    if (e >= cnt) return t_unit + (e - cnt);             // a drafted row
+    if (idx_value < 0 || idx_value >= t_unit) {
       record_error(p.status, BD_ERR_INVALID_ARG);
       return -1;                                         // skipped
     }
@@ -136,7 +141,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
       const int r = c / CH, ch = c % CH;
       const int pos = rowpos[b * kDRows + r];
       const bool live = r < nrows && pos >= 0;   // others zero-filled (0 * garbage could be NaN in P V)
-      const bool drafted = live && pos >= p.t_ctx;
+      const bool drafted = live && pos >= t_unit;
       if ((part == 0 && drafted) || (part == 1 && !drafted)) continue;
       const uint32_t off = sw128_offset(r, ch * 8, HALF_BYTES);
       const size_t src = (size_t)max(pos, 0) * D + ch * 8;
@@ -291,6 +296,8 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.budget = budget;
   p.step_j = step_j;
   p.t_ctx = s.t_ctx;
+  p.seq_lens = s.seq_lens;
+  p.h_kv = s.h_kv;
   p.t_cap = s.t_cap;
   p.n_split = plan.n_split;
   p.rows_per_split = plan.rows_per_split;

@@ -45,7 +45,8 @@ size_t verify_partials_bytes(const bd_shape& s, const VerifyPlan& plan);
 // q/o/lse as in bd_verify_attn; ws_region points at the op region, counters/status into ws.
 cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, const void* q,
                           const void* k_cache, const void* v_cache, void* o_out, float* lse_out,
-                          void* ws_region, int* counters, int* status, cudaStream_t stream);
+                          void* ws_region, int* counters, int* status, cudaStream_t stream,
+                          int len_offset = 0);
 
 // ---------------------------------------------------------------------------- draft
 struct DraftPlan {
@@ -101,6 +102,8 @@ cudaError_t launch_argmax(const void* logits, bool bf16, int rows, int vocab, in
 cudaError_t launch_accept(int batch, int gamma, const int32_t* draft_tokens, const int32_t* verify_tokens,
                           int32_t* n_accept, int32_t* emit, cudaStream_t stream);
 size_t advance_smem(int window, int head_dim);
+cudaError_t launch_write_rows(const bd_shape& s, int n_rows, const void* k_rows, const void* v_rows, void* k_cache,
+                              void* v_cache, cudaStream_t stream);
 cudaError_t launch_advance(const bd_shape& s, int window, int n_q, const int32_t* n_accept, const void* q_verify,
                            const float* verify_lse, void* q_window, float* window_lse, int32_t* idx, int32_t* count,
                            int capacity, int32_t* advance_out, cudaStream_t stream);

@@ -46,6 +46,8 @@ struct ScoreParams {
   int n_acc;                    // accumulators: tile i uses i % n_acc; epilogue group i % 2
   uint32_t tmem_cols;
   float scale_log2;
+  const int32_t* seq_lens;      // per-sequence context lengths [batch] or null (all t_ctx)
+  int h_kv;
 };
 
 template <int D, int STAGES, int NQB>
@@ -193,12 +195,19 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     const int ep_tid = (warp - 2 - 4 * grp) * 32 + lane;
     float* lse2_s = reinterpret_cast<float*>(smem + 1024 + grp * 2304);   // [288] -lse * log2(e)
     int* pw_s = reinterpret_cast<int*>(smem + 1024 + grp * 2304 + 1152);  // [288]
-    const int win0 = p.t_ctx - p.window;        // position of window row 0
+    int win0 = p.t_ctx - p.window;              // position of window row 0 (of the current unit)
+    int mid_end = p.mid_end;                    // end of the current unit's middle
     int cur_unit = -1;
     for (int i = grp; i < n; i += 2) {
       const int g = first + i;
       const int unit = g / p.tiles_per_unit, tt = g % p.tiles_per_unit;
       if (unit != cur_unit) {
+        if (p.seq_lens) {
+          const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, ep_tid == 0 ? p.status : nullptr);
+          if (t_u < p.window && ep_tid == 0) record_error(p.status, BD_ERR_INVALID_ARG);
+          win0 = t_u - p.window;
+          mid_end = t_u - (p.t_ctx - p.mid_end);
+        }
         named_bar(1 + grp, 128);
         for (int c = ep_tid; c < 288; c += 128) {
           const bool real = c < p.nq_rows;
@@ -257,7 +266,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&tempty_bar[acc]);
-      if (key < p.mid_end) p.score[(size_t)unit * p.n_mid_pad + (key - p.n_sink)] = (sum0 + sum1) + (sum2 + sum3);
+      if (key < mid_end) p.score[(size_t)unit * p.n_mid_pad + (key - p.n_sink)] = (sum0 + sum1) + (sum2 + sum3);
     }
   }
 
@@ -276,7 +285,18 @@ struct TopkParams {
   int t_ctx, budget, n_sink, n_recent, chunk, n_mid_pad;
   int keep_all;            // budget >= t_ctx
   int smem_items;          // item values staged in shared memory when n_items <= smem_items
+  const int32_t* seq_lens; // per-sequence context lengths [batch] or null (all t_ctx)
+  int h_kv;
+  int* status;
 };
+
+// A unit whose context fits the budget keeps every position (the B >= T rule).
+__device__ __forceinline__ bool topk_keep_all(const TopkParams& p, int unit, int t_u, int32_t* out) {
+  if (!p.keep_all && p.budget < t_u) return false;
+  for (int i = threadIdx.x; i < p.budget; i += blockDim.x) out[i] = i < t_u ? i : -1;
+  if (threadIdx.x == 0) p.count_out[unit] = t_u;
+  return true;
+}
 
 // Exclusive scan of one value per warp (32 warps), result broadcast through smem.
 __device__ __forceinline__ uint32_t warp_totals_exclusive(uint32_t v, uint32_t* wsum, uint32_t* total) {
@@ -311,12 +331,9 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_kernel(const TopkParams 
   const int unit = blockIdx.x;
   int32_t* out = p.idx_out + (size_t)unit * p.budget;
 
-  if (p.keep_all) {
-    for (int i = tid; i < p.budget; i += kTopkThreads) out[i] = i < p.t_ctx ? i : -1;
-    if (tid == 0) p.count_out[unit] = p.t_ctx;
-    return;
-  }
-  const int lo = p.n_sink, hi = p.t_ctx - p.n_recent;
+  const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
+  if (topk_keep_all(p, unit, t_u, out)) return;
+  const int lo = p.n_sink, hi = t_u - p.n_recent;
   const int s = p.chunk;
   const int free = p.budget - p.n_sink - p.n_recent;
   const int c_first = lo / s;
@@ -616,10 +633,12 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_token_kernel(const TopkP
   allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int unit = blockIdx.x;
-  const int lo = p.n_sink, hi = p.t_ctx - p.n_recent, n = hi - lo;
+  const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
+  int32_t* out = p.idx_out + (size_t)unit * p.budget;
+  if (topk_keep_all(p, unit, t_u, out)) return;
+  const int lo = p.n_sink, hi = t_u - p.n_recent, n = hi - lo;
   const int k = p.budget - p.n_sink - p.n_recent;
   const float* sc = p.score + (size_t)unit * p.n_mid_pad;
-  int32_t* out = p.idx_out + (size_t)unit * p.budget;
 
   // ---- stage the scores, min and max
   float lmin = INFINITY, lmax = -INFINITY;
@@ -895,10 +914,12 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
   allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int unit = blockIdx.x;
-  const int lo = p.n_sink, hi = p.t_ctx - p.n_recent, n = hi - lo;
+  const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
+  int32_t* out = p.idx_out + (size_t)unit * p.budget;
+  if (topk_keep_all(p, unit, t_u, out)) return;
+  const int lo = p.n_sink, hi = t_u - p.n_recent, n = hi - lo;
   const int k = p.budget - p.n_sink - p.n_recent;
   const float* sc = p.score + (size_t)unit * p.n_mid_pad;
-  int32_t* out = p.idx_out + (size_t)unit * p.budget;
   const int w0 = warp * ROWS * 32;
 
   // ---- the thread's scores (fp32 bits; non-negative, so their order is the bits' order)
@@ -1221,7 +1242,7 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
       bd_shape ls = s;
       ls.t_ctx = s.t_ctx - window;
       err = launch_verify(ls, plan.lse_plan, window, q_window, k_cache, nullptr, nullptr, lse_buf,
-                          region + plan.score_bytes + plan.lse_bytes, counters, status, stream);
+                          region + plan.score_bytes + plan.lse_bytes, counters, status, stream, -window);
       if (err != cudaSuccess) return err;
       lse = lse_buf;
     }
@@ -1249,6 +1270,8 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
     p.n_acc = plan.n_acc;
     p.tmem_cols = plan.tmem_cols;
     p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
+    p.seq_lens = s.seq_lens;
+    p.h_kv = s.h_kv;
     void* fn = score_fn(s.head_dim, plan.nq_pad).fn;
     err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
     if (err != cudaSuccess) return err;
@@ -1267,6 +1290,9 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
   tp.chunk = chunk;
   tp.n_mid_pad = plan.n_mid_pad;
   tp.keep_all = plan.keep_all ? 1 : 0;
+  tp.seq_lens = s.seq_lens;
+  tp.h_kv = s.h_kv;
+  tp.status = status;
   void* targs[] = {&tp};
   const int free = budget - n_sink - n_recent;
   if (!plan.keep_all && plan.need_scores && chunk == 1 && free < plan.n_mid && plan.n_mid <= 16 * kTopkThreads) {

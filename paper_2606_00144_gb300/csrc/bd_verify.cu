@@ -36,6 +36,9 @@ struct VerifyParams {
   float* lse_part;     // [units][max_seg][nq_rows]
   int* counters;       // [units]
   int* status;
+  const int32_t* seq_lens;  // per-sequence context lengths [batch] or null (all t_ctx)
+  int h_kv;
+  int len_offset;      // added to every length (the window LSE pass runs at T - W)
   int n_q, nq_rows, t_ctx, tiles_per_unit, total_tiles, max_seg;
   int seg_cost;        // virtual tiles charged for each unit a CTA starts (see verify_plan)
   int vtiles_per_cta;  // contiguous range of the virtual tile list per CTA
@@ -117,7 +120,13 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
       tma_prefetch_map(&kmap);
       if (WITH_V) tma_prefetch_map(&vmap);
       int issued = 0;
+      // with per-sequence lengths any tile may hold some sequence's block rows (written by
+      // the preceding kernels): wait before the first load
       bool waited = false;
+      if (p.seq_lens) {
+        grid_dependency_wait();
+        waited = true;
+      }
       for (int t = 0; t < ntiles; ++t) {
         const int s = t % STAGES;
         if (t >= STAGES && !mbar_wait(&empty_bar[s], ((t / STAGES) & 1) ^ 1, p.status, abort_flag)) break;
@@ -155,19 +164,21 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   const int nq = p.nq_rows;
   constexpr int NCT = kVConsumers * 32;          // consumer threads
   int lim[NT][2];                                // last visible key of each of this thread's columns
-#pragma unroll
-  for (int nt = 0; nt < NT; ++nt)
-#pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      const int col = 8 * (wq * NT + nt) + 2 * tig + e;
-      lim[nt][e] = col < nq ? p.t_ctx + col % p.n_q : -1;
-    }
 
   bool alive = true;   // false once this warp's wait gave up (the abort flag is then set)
   int t = 0;
   for (int seg_start = g0; seg_start < g1;) {
     const int unit = seg_start / p.tiles_per_unit;
     const int seg_end = min(g1, (unit + 1) * p.tiles_per_unit);
+    const int t_unit = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx - p.len_offset, tid == 0 ? p.status : nullptr) +
+                       p.len_offset;
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const int col = 8 * (wq * NT + nt) + 2 * tig + e;
+        lim[nt][e] = col < nq ? t_unit + col % p.n_q : -1;
+      }
     uint32_t bq[NT][D / 16][2];
     WarpAttn<D, NT, WITH_V>::load_q(bq, p.q + (size_t)unit * nq * D, nq, wq * NT, lane);
     WarpAttn<D, NT, WITH_V> wa;
@@ -345,7 +356,7 @@ size_t verify_partials_bytes(const bd_shape& s, const VerifyPlan& plan) {
 
 cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, const void* q,
                           const void* k_cache, const void* v_cache, void* o_out, float* lse_out,
-                          void* ws_region, int* counters, int* status, cudaStream_t stream) {
+                          void* ws_region, int* counters, int* status, cudaStream_t stream, int len_offset) {
   const int units = s.batch * s.h_kv;
   CUtensorMap kmap, vmap;
   cudaError_t err = make_cache_map(&kmap, k_cache, units, s.t_cap, s.t_ctx + n_q, s.head_dim, kVKeys);
@@ -368,6 +379,9 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.n_q = n_q;
   p.nq_rows = plan.nq_rows;
   p.t_ctx = s.t_ctx;
+  p.seq_lens = s.seq_lens;
+  p.h_kv = s.h_kv;
+  p.len_offset = len_offset;
   p.tiles_per_unit = plan.tiles_per_unit;
   p.total_tiles = plan.total_tiles;
   p.seg_cost = plan.seg_cost;

@@ -15,8 +15,11 @@ class SpecStep:
     on one stream are ordered)."""
 
     def __init__(self, batch, h_q, h_kv, head_dim, t_ctx, t_cap, budget, n_sink, n_recent,
-                 window=32, gamma=5, chunk=1, device="cuda"):
-        self.shape = B.make_shape(batch, h_q, h_kv, head_dim, t_ctx, t_cap)
+                 window=32, gamma=5, chunk=1, device="cuda", seq_lens=None):
+        """seq_lens: optional int32 device tensor [batch] of per-sequence context lengths
+        (t_ctx is then the longest; bd_advance moves them on the device)."""
+        self.seq_lens = seq_lens
+        self.shape = B.make_shape(batch, h_q, h_kv, head_dim, t_ctx, t_cap, seq_lens)
         self.budget, self.n_sink, self.n_recent = budget, n_sink, n_recent
         self.window, self.gamma, self.chunk = window, gamma, chunk
         self.ws = B.Workspace.for_step(self.shape, budget, window, gamma, device)
@@ -67,6 +70,8 @@ class SpecStep:
     def window_lse(self, k_cache, q_win, out=None, stream=None):
         """LSE of the window queries over their causal prefixes, computed by the verify
         kernel (what a previous verify / prefill step leaves behind for carry mode)."""
+        if self.seq_lens is not None:
+            raise NotImplementedError("window_lse with per-sequence lengths: use bd_select_budget's self mode")
         sh = B.make_shape(self.shape.batch, self.shape.h_q, self.shape.h_kv, self.shape.head_dim,
                           self.shape.t_ctx - self.window, self.shape.t_cap)
         if out is None:

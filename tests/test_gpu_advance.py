@@ -39,13 +39,13 @@ def test_advance_matches_oracle(n_acc, window, n_q):
     dev = {k: v.cuda() for k, v in dict(q_win=q_win, q_ver=q_ver, lse_win=lse_win, lse_ver=lse_ver, idx=idx,
                                         count=count).items()}
     n_dev = torch.tensor(n_acc, dtype=torch.int32, device="cuda")
-    out = torch.zeros(1, dtype=torch.int32, device="cuda")
+    out = torch.zeros(b, dtype=torch.int32, device="cuda")
     shape = bd.make_shape(b, hq, hkv, d, t, t + n_q)
     bd.bd_advance(shape, window, n_q, n_dev, dev["q_ver"], dev["lse_ver"], dev["q_win"], dev["lse_win"], dev["idx"],
                   dev["count"], out)
     torch.cuda.synchronize()
     a = oracle.batch_advance(np.array(n_acc), n_q)
-    assert int(out.item()) == a
+    assert out.cpu().tolist() == [a] * b
     q_ref, l_ref = oracle.advance_window(f64(q_win), lse_win.double().numpy(), f64(q_ver), lse_ver.double().numpy(), a)
     assert np.array_equal(f64(dev["q_win"]), q_ref)                     # a copy: bit-exact
     assert np.array_equal(dev["lse_win"].cpu().double().numpy(), l_ref)
@@ -78,7 +78,7 @@ def test_multistep_carry_selection_on_the_slid_window():
     cnt = torch.empty(b, hkv, dtype=torch.int32, device="cuda")
     vo = torch.empty(b, hq, gamma + 1, d, dtype=torch.bfloat16, device="cuda")
     vl = torch.empty(b, hq, gamma + 1, dtype=torch.float32, device="cuda")
-    adv = torch.zeros(1, dtype=torch.int32, device="cuda")
+    adv = torch.zeros(b, dtype=torch.int32, device="cuda")
     for step in range(steps):
         shape = bd.make_shape(b, hq, hkv, d, t, cap)
         ws = bd.Workspace.for_step(shape, budget, W, gamma)
@@ -103,7 +103,7 @@ def test_multistep_carry_selection_on_the_slid_window():
         bd.bd_advance(shape, W, gamma + 1, torch.from_numpy(n_acc).int().cuda(), q_ver, vl, q_win, lse_win, None,
                       None, adv)
         torch.cuda.synchronize()
-        a = int(adv.item())
+        a = int(adv[0].item())
         assert a == oracle.batch_advance(n_acc, gamma + 1)
         t += a
         assert torch.equal(q_win, q_all[:, :, t - W: t])
@@ -140,7 +140,7 @@ def test_amortised_loop_view_grows_by_the_settled_rows():
     vl = torch.empty(b, hq, gamma + 1, dtype=torch.float32, device="cuda")
     do = torch.empty(b, hq, d, dtype=torch.bfloat16, device="cuda")
     dl = torch.empty(b, hq, dtype=torch.float32, device="cuda")
-    adv = torch.zeros(1, dtype=torch.int32, device="cuda")
+    adv = torch.zeros(b, dtype=torch.int32, device="cuda")
     for step in range(steps):
         shape = bd.make_shape(b, hq, hkv, d, t, cap_rows)
         ws = bd.Workspace.for_step(shape, capacity, W, gamma)
@@ -158,7 +158,7 @@ def test_amortised_loop_view_grows_by_the_settled_rows():
         bd.bd_advance(shape, W, gamma + 1, torch.from_numpy(n_acc).int().cuda(), q_ver, vl, q_win, lse_win, idx,
                       cnt, adv)
         torch.cuda.synchronize()
-        a = int(adv.item())
+        a = int(adv[0].item())
         i_ref, c_ref, full = oracle.append_view(idx_h, cnt_h, t, a, capacity)
         assert not full
         assert idx.cpu().numpy().tolist() == i_ref.tolist() and cnt.cpu().numpy().tolist() == c_ref.tolist()
