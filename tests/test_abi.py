@@ -172,3 +172,11 @@ def test_write_block_rows_validation(lib):
     assert f(ctypes.byref(shape()), 6, A + 8, A, A, A, None) == MISALIGNED
     assert f(ctypes.byref(shape()), 6, A, A, None, A, None) == INVALID
     assert f(ctypes.byref(shape(head_dim=96)), 6, A, A, A, A, None) == UNSUPPORTED
+
+
+def test_seq_lens_pointer_is_checked(lib):
+    s = shape()
+    s.seq_lens = A + 2
+    assert verify(lib, s) == MISALIGNED
+    s.seq_lens = A
+    assert verify(lib, s, n_q=0) == INVALID            # the other checks still run
