@@ -12,7 +12,7 @@
 //                 warp 1   one lane issues tcgen05.mma into four fp32 TMEM accumulators
 //                          (two when the window rows need more columns) and commits to
 //                          the smem/TMEM barriers;
-//                 warps 2-9 epilogue (two groups of 4, alternate tiles): tcgen05.ld,
+//                 warps 2-17 epilogue (four groups of 4, every fourth tile): tcgen05.ld,
 //                          packed f32x2 FMA, ex2 (MUFU), packed row sums, coalesced store.
 // topk_kernel   one CTA per (sequence, KV head), scores staged in shared memory: a linear
 //               histogram between the min and max score finds the bin holding the k-th
@@ -27,9 +27,9 @@
 namespace bd {
 
 constexpr int kSKeys = 128;          // keys per tile (UMMA M)
-constexpr int kSThreads = 320;       // producer, MMA, 2 x 4 epilogue warps
+constexpr int kSThreads = 576;       // producer, MMA, 4 x 4 epilogue warps
 constexpr int kMaxAcc = 4;           // TMEM accumulators (<= 512 columns)
-constexpr int kSQOffset = 8192;      // shared-memory offset of the window-query tiles
+constexpr int kSQOffset = 12288;     // shared-memory offset of the window-query tiles
 constexpr int kTopkThreads = 1024;
 constexpr int kTopkSmemBytes = 200 * 1024;   // item values staged in shared memory up to this size
 constexpr int kBins = 4096;                   // linear histogram bins of the value range
@@ -43,7 +43,7 @@ struct ScoreParams {
   int nq_rows, nq_pad, window, t_ctx, n_sink, mid_end, n_mid_pad;
   int tiles_per_unit, total_tiles, tiles_per_cta;
   int acc_stride;               // TMEM columns between accumulators
-  int n_acc;                    // accumulators: tile i uses i % n_acc; epilogue group i % 2
+  int n_acc;                    // accumulators: tile i uses i % n_acc; epilogue group i % 4
   uint32_t tmem_cols;
   float scale_log2;
   const int32_t* seq_lens;      // per-sequence context lengths [batch] or null (all t_ctx)
@@ -190,7 +190,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     // ---------------------------------------------------------------- epilogue (2 groups of 4 warps)
     grid_dependency_wait();                      // the window LSE is carried from earlier kernels
     allow_dependent_launch();
-    const int grp = (warp - 2) >> 2;            // group 0: warps 2-5, group 1: warps 6-9; tiles i % 2 == grp
+    const int grp = (warp - 2) >> 2;            // group g: warps 2+4g .. 5+4g; tiles i % 4 == g
     const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
     const int ep_tid = (warp - 2 - 4 * grp) * 32 + lane;
     float* lse2_s = reinterpret_cast<float*>(smem + 1024 + grp * 2304);   // [288] -lse * log2(e)
@@ -198,7 +198,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     int win0 = p.t_ctx - p.window;              // position of window row 0 (of the current unit)
     int mid_end = p.mid_end;                    // end of the current unit's middle
     int cur_unit = -1;
-    for (int i = grp; i < n; i += 2) {
+    for (int i = grp; i < n; i += 4) {
       const int g = first + i;
       const int unit = g / p.tiles_per_unit, tt = g % p.tiles_per_unit;
       if (unit != cur_unit) {
