@@ -180,3 +180,24 @@ def test_seq_lens_pointer_is_checked(lib):
     assert verify(lib, s) == MISALIGNED
     s.seq_lens = A
     assert verify(lib, s, n_q=0) == INVALID            # the other checks still run
+
+
+def test_plain_c_consumer(lib, tmp_path):
+    # the header compiles as C and the library links and answers from a C program
+    import shutil
+    import subprocess
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no C compiler")
+    here = os.path.dirname(__file__)
+    exe = tmp_path / "consumer"
+    lib_dir = os.path.dirname(bd.LIB_PATH)
+    subprocess.run([gcc, "-std=c99", "-Wall", "-Werror", "-I", os.path.dirname(HEADER),
+                    os.path.join(here, "c_abi_consumer.c"), "-o", str(exe), "-L", lib_dir, "-lbudgetdraft",
+                    f"-Wl,-rpath,{lib_dir}"], check=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split("\n")
+    assert out[0] == "workspace_size 0"
+    assert out[1] == f"verify {UNSUPPORTED}"
+    assert out[2] == f"argmax {INVALID}"
+    assert out[3] == f"accept_empty {BD_OK}"
+    assert out[4] == "strerror " + bd.bd_strerror(MISALIGNED)
