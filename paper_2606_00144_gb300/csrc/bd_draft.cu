@@ -6,16 +6,18 @@
 // KV head) unit, each CTA one slice of its entry list:
 //   1. count and the slice's indices are fetched together (indices speculatively, before
 //      count is known);
-//   2. rows are gathered with 16-byte cp.async straight into the 128-byte swizzled layout
-//      (unused rows zero-filled) and the four warps run the mma.sync sub-tile code shared
-//      with the verify kernel (bd_attn_warp.cuh), the G heads of the GQA group forming one
-//      n8 query tile;
+//   2. rows (80 per CTA) are gathered with 16-byte cp.async straight into the 128-byte
+//      swizzled layout (unused rows zero-filled) and the five warps run the mma.sync
+//      sub-tile code shared with the verify kernel (bd_attn_warp.cuh), the G heads of the
+//      GQA group forming one n8 query tile;
 //   3. every CTA stores its normalised partial straight into the shared memory of the
 //      cluster's rank-0 CTA (distributed shared memory); after one cluster barrier rank 0
 //      merges them (log-sum-exp) from its own shared memory and writes the bf16 output:
 //      no global partials, fences or atomics.
 // Launched with programmatic dependent launch: the grid-dependency wait is the first thing
-// a CTA does, and the next kernel may be scheduled as soon as every CTA has passed it.
+// a CTA does, except with BD_DRAFT_VIEW_READY, where the selected rows (and the unit's
+// context length) are read and gathered first and only the queries and the drafted rows
+// after the wait.  The next kernel may be scheduled as soon as every CTA has passed it.
 #include <cooperative_groups.h>
 
 #include <algorithm>

@@ -14,11 +14,14 @@
 //                          the smem/TMEM barriers;
 //                 warps 2-17 epilogue (four groups of 4, every fourth tile): tcgen05.ld,
 //                          packed f32x2 FMA, ex2 (MUFU), packed row sums, coalesced store.
-// topk_kernel   one CTA per (sequence, KV head), scores staged in shared memory: a linear
-//               histogram between the min and max score finds the bin holding the k-th
-//               largest; that bin's few items are ranked exactly by (score desc, position
-//               asc) (4-pass radix select on the fp32 bits when the bin is crowded); then an
-//               ascending compaction (warp ballots + block scan) with sinks and recents.
+// top-B         one CTA per (sequence, KV head): a linear histogram between the min and
+//               max score finds the bin holding the k-th largest; that bin's few items are
+//               ranked exactly by (score desc, position asc) (4-pass radix select on the
+//               fp32 bits when the bin is crowded); then an ascending compaction (warp
+//               ballots + block scan) with sinks and recents.  Three kernels of that
+//               method: topk_rows_kernel (token level, up to 16K middle positions, every
+//               score in registers), topk_token_kernel (token level, up to 32K, scores in
+//               shared memory) and topk_kernel (chunk level and longer contexts).
 #include <algorithm>
 
 #include "bd_common.cuh"

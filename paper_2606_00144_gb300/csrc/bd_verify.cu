@@ -3,15 +3,18 @@
 // [0, t_ctx + i] (causal inside the block).
 //
 // Persistent, stream-K scheduled: the (unit, 64-key tile) pairs of all (sequence, KV head)
-// units form one list that is cut into equal contiguous ranges, one per CTA, so every SM
-// streams the same number of bytes whatever the batch.  A range covers one or two units;
-// each piece of a unit ("segment") ends in a normalised partial (o, lse), and the last
-// CTA to finish a unit merges its segments (log-sum-exp) into the final bf16 output.
+// units form one list that is cut into contiguous ranges, one per CTA, of equal cost: each
+// unit's tiles are preceded by a few virtual tiles that stand for the cost of starting a
+// unit, so every SM streams about the same time whatever the batch.  A range covers one or
+// two units; each piece of a unit ("segment") ends in a normalised partial (o, lse), and
+// the last CTA to finish a unit merges its segments (log-sum-exp) into the final bf16
+// output, staging the partials in shared memory with cp.async (one round trip).
 //   warp 4      TMA producer: 64-key K (and V) tiles, 128-byte swizzle, 5-stage ring,
 //               streaming straight across segment boundaries.  Context rows [0, t_ctx)
 //               are streamed before the grid-dependency wait (they are not written by
 //               the preceding kernel); the wait comes before the first tile that holds
-//               the block's own rows;
+//               the block's own rows (before the first load when per-sequence lengths
+//               are given: any tile may then hold some sequence's block rows);
 //   warps 0..3  consumers on mma.sync (bd_attn_warp.cuh): the GQA group's packed query
 //               rows are the N side of S^T = K Q^T.
 #include <algorithm>
