@@ -503,6 +503,12 @@ def e2e_measure(step, args, world, bytes_per_step):
                    "double-buffered) around SpecStep through the C ABI, one CUDA graph"}
 
 
+def code_lines(text):
+    """The source without whole-line comments and blank lines: what the kernel is built from
+    (a comment edit leaves the profiled counters valid)."""
+    return "\n".join(ln.strip() for ln in text.splitlines() if ln.strip() and not ln.strip().startswith("//"))
+
+
 def profiled_traffic(kernel, workload, sources):
     """dram bytes read + written per launch from the committed ncu summary, or None when
     the summary is missing or was taken on other kernel sources than the ones built now."""
@@ -514,8 +520,8 @@ def profiled_traffic(kernel, workload, sources):
         return None
     h = hashlib.sha256()
     for f in sources:
-        with open(os.path.join(ROOT, "paper_2606_00144_gb300", "csrc", f), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2606_00144_gb300", "csrc", f)) as fh:
+            h.update(code_lines(fh.read()).encode())
     fields = dict(ln.split(":", 1) for ln in text.splitlines() if ln.startswith(("source_sha256:", "traffic_bytes")))
     if fields.get("source_sha256", "").split()[0:1] != [h.hexdigest()[:16]]:
         return None
