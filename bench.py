@@ -181,12 +181,13 @@ class Step:
     `share`: another Step whose inputs and carried LSE this one reuses (a policy variant on
     the same data)."""
 
-    def __init__(self, wl, budget, n_recent, sel_mode, device, share=None, n_sink=None, chunk=1):
+    def __init__(self, wl, budget, n_recent, sel_mode, device, share=None, n_sink=None, chunk=1, seq_lens=None):
         import paper_2606_00144_gb300 as bd
         self.wl, self.budget, self.n_recent, self.sel_mode = wl, budget, n_recent, sel_mode
         self.n_sink = wl.n_sink if n_sink is None else n_sink
         self.steps = [bd.SpecStep(wl.batch, wl.h_q, wl.h_kv, wl.head_dim, wl.t_ctx, wl.t_cap, budget, self.n_sink,
-                                  n_recent, wl.window, wl.gamma, chunk, device) for _ in range(wl.layers)]
+                                  n_recent, wl.window, wl.gamma, chunk, device, seq_lens)
+                      for _ in range(wl.layers)]
         if share is not None:
             self.layers, self.lse = share.layers, share.lse
             return
@@ -457,6 +458,18 @@ def extras(step, args):
                          "GB/s": round(pb / (us * 1e-6) / 1e9, 1)})
             del v
         out["chunk_policy"] = rows
+        # a ragged batch: per-sequence context lengths spread over the lower quarter of T (the
+        # same cache, window and carried LSE; the timing does not depend on their values)
+        lens = [wl.t_ctx - (wl.t_ctx // 4) * i // max(1, wl.batch - 1) for i in range(wl.batch)]
+        lens_d = torch.tensor(lens, dtype=torch.int32, device="cuda")
+        v = Step(wl, step.budget, step.n_recent, step.sel_mode, "cuda", share=step, seq_lens=lens_d)
+        us = time_per_step(v.run, n, gs)
+        row, units_per_seq = wl.head_dim * 2, wl.h_kv
+        rb = sum(((t - wl.n_sink - step.n_recent) + (min(step.budget, t) + wl.gamma) * 2 + (t + wl.gamma + 1) * 2)
+                 * row * units_per_seq for t in lens) * wl.layers
+        out["ragged_lengths"] = {"seq_lens": lens, "us_per_step": round(us, 2), "GB/s": round(rb / (us * 1e-6) / 1e9, 1),
+                                 "bytes_per_step": rb}
+        del v
     out["note"] = "each timed over %d graphed steps outside the headline timed region" % n
     return out
 

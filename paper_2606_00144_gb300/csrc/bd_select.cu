@@ -53,7 +53,9 @@ struct ScoreParams {
   int h_kv;
 };
 
-template <int D, int STAGES, int NQB>
+// RAGGED: per-sequence lengths (the tile layout is built on the device); a separate
+// instance, since the uniform kernel measured 6 us slower with the ragged branches inlined.
+template <int D, int STAGES, int NQB, bool RAGGED>
 __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p,
                                                              const __grid_constant__ CUtensorMap kmap,
                                                              const __grid_constant__ CUtensorMap qmap) {
@@ -75,9 +77,65 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
   uint8_t* kstage = qbuf + NQB * qbytes;                       // STAGES x KTILE (1024-aligned)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int first = blockIdx.x * p.tiles_per_cta;
-  const int n = max(0, min(p.tiles_per_cta, p.total_tiles - first));
   const int n_acc = p.n_acc;
+  const int n_units = p.total_tiles / p.tiles_per_unit;
+  // per-sequence lengths: every CTA lays out the units' middle tiles itself (prefix table
+  // after the K stages; the lengths may come from the preceding kernel, so after the
+  // dependency wait) and cuts the tile list over the actual tiles
+  int* spref = reinterpret_cast<int*>(kstage + STAGES * KTILE);   // [units + 1]
+  int total = p.total_tiles, tpc = p.tiles_per_cta;
+  if (RAGGED) {
+    grid_dependency_wait();
+    int* wtot = reinterpret_cast<int*>(smem + 1024);
+    const int per = (n_units + kSThreads - 1) / kSThreads;
+    const int u0 = min(n_units, tid * per), u1 = min(n_units, u0 + per);
+    const int tail = p.t_ctx - p.mid_end;            // recent positions
+    auto tiles_of = [&](int u) {
+      const int t_u = unit_context(p.seq_lens, u, p.h_kv, p.t_ctx, nullptr);
+      return (max(0, t_u - tail - p.n_sink) + kSKeys - 1) / kSKeys;
+    };
+    int sum = 0;
+    for (int u = u0; u < u1; ++u) sum += tiles_of(u);
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    if (lane == 31) wtot[warp] = incl;
+    __syncthreads();
+    int run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += wtot[w];
+    for (int u = u0; u < u1; ++u) {
+      spref[u] = run;
+      run += tiles_of(u);
+    }
+    if (tid == kSThreads - 1) spref[n_units] = run;
+    __syncthreads();
+    total = spref[n_units];
+    tpc = (total + (int)gridDim.x - 1) / (int)gridDim.x;
+  }
+  const int first = blockIdx.x * tpc;
+  const int n = max(0, min(tpc, total - first));
+  // (unit, tile within the unit's middle) of tile g of the list
+  auto locate = [&](int g, int& unit, int& tt) {
+    if (!RAGGED) {
+      unit = g / p.tiles_per_unit;
+      tt = g - unit * p.tiles_per_unit;
+      return;
+    }
+    int lo = 0, hi = n_units - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (spref[mid] <= g) lo = mid;
+      else hi = mid - 1;
+    }
+    unit = lo;
+    tt = g - spref[lo];
+  };
+  auto last_of_unit = [&](int g, int unit) {
+    return RAGGED ? g + 1 == spref[unit + 1] : (g + 1) % p.tiles_per_unit == 0;
+  };
 
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -115,7 +173,8 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     int cur_unit = -1, qcount = 0;
     for (int i = 0; i < n; ++i) {
       const int g = first + i;
-      const int unit = g / p.tiles_per_unit, tt = g % p.tiles_per_unit;
+      int unit, tt;
+      locate(g, unit, tt);
       if (unit != cur_unit) {
         const int qs = qcount % NQB;
         bool ok = true;
@@ -157,8 +216,9 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       int cur_unit = -1, qcount = 0;
       for (int i = 0; i < n; ++i) {
         const int g = first + i;
-        const int unit = g / p.tiles_per_unit;
-        const bool last_of_unit = (i == n - 1) || ((g + 1) / p.tiles_per_unit != unit);
+        int unit, tt;
+        locate(g, unit, tt);
+        const bool unit_ends = (i == n - 1) || last_of_unit(g, unit);
         if (unit != cur_unit) {
           if (!mbar_wait(&qfull_bar[qcount % NQB], (qcount / NQB) & 1, p.status, abort_flag)) break;
           cur_unit = unit;
@@ -183,7 +243,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
         }
         tc_commit(&empty_bar[s]);
         tc_commit(&tfull_bar[acc]);
-        if (last_of_unit) tc_commit(&qempty_bar[qs]);
+        if (unit_ends) tc_commit(&qempty_bar[qs]);
       }
       // every MMA this thread issued has completed before TMEM is released
       tc_commit(drain_bar);
@@ -203,9 +263,10 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     int cur_unit = -1;
     for (int i = grp; i < n; i += 4) {
       const int g = first + i;
-      const int unit = g / p.tiles_per_unit, tt = g % p.tiles_per_unit;
+      int unit, tt;
+      locate(g, unit, tt);
       if (unit != cur_unit) {
-        if (p.seq_lens) {
+        if (RAGGED) {
           const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, ep_tid == 0 ? p.status : nullptr);
           if (t_u < p.window && ep_tid == 0) record_error(p.status, BD_ERR_INVALID_ARG);
           win0 = t_u - p.window;
@@ -1167,7 +1228,7 @@ struct ScoreKernel {
 // Two window-query buffers (a unit switch inside a CTA's range does not stall) and four
 // K stages when they fit, else one Q buffer and as many stages as fit (measured: a fifth
 // stage does not speed the kernel up).
-ScoreKernel score_fn(int d, int nq_pad) {
+ScoreKernel score_fn(int d, int nq_pad, bool ragged) {
   const size_t qbytes = (size_t)nq_pad * d * 2;
   const size_t kt = (size_t)kSKeys * d * 2;
   const size_t budget = 227 * 1024 - 1024 - kSQOffset;
@@ -1176,8 +1237,10 @@ ScoreKernel score_fn(int d, int nq_pad) {
     nqb = 1;
     if (qbytes + 5 * kt <= budget) stages = 5;
   }
-#define BD_SK(DD, ST, NB) \
-  if (d == DD && stages == ST && nqb == NB) return {reinterpret_cast<void*>(&score_kernel<DD, ST, NB>), ST, NB};
+#define BD_SK(DD, ST, NB)                                                                              \
+  if (d == DD && stages == ST && nqb == NB)                                                              \
+    return {ragged ? reinterpret_cast<void*>(&score_kernel<DD, ST, NB, true>)                            \
+                   : reinterpret_cast<void*>(&score_kernel<DD, ST, NB, false>), ST, NB};
   BD_SK(64, 5, 1) BD_SK(64, 4, 2) BD_SK(64, 4, 1) BD_SK(128, 5, 1) BD_SK(128, 4, 2) BD_SK(128, 4, 1)
 #undef BD_SK
   return {nullptr, 0, 0};
@@ -1203,7 +1266,7 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   const int free = budget - n_sink - n_recent;
   plan->need_scores = !plan->keep_all && plan->n_mid > 0 && free / chunk > 0;
   if (plan->nq_pad > 256) return false;
-  const ScoreKernel sk = score_fn(s.head_dim, plan->nq_pad);
+  const ScoreKernel sk = score_fn(s.head_dim, plan->nq_pad, s.seq_lens != nullptr);
   if (!sk.fn) return false;
   plan->tiles_per_unit = (plan->n_mid + kSKeys - 1) / kSKeys;
   plan->total_tiles = plan->tiles_per_unit * units;
@@ -1217,6 +1280,10 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   plan->tmem_cols = pow2_at_least((uint32_t)plan->n_acc * acc_stride);
   plan->smem_bytes = 1024 + kSQOffset + (size_t)sk.nqb * plan->nq_pad * s.head_dim * 2 +
                      (size_t)sk.stages * kSKeys * s.head_dim * 2;
+  if (s.seq_lens) {   // the units' tile table of per-sequence lengths
+    plan->smem_bytes += align_up((size_t)(units + 1) * 4, 16);
+    if (plan->smem_bytes > 227 * 1024) return false;
+  }
   plan->score_bytes = plan->need_scores ? align_up((size_t)units * plan->n_mid_pad * 4, 256) : 0;
   plan->lse_bytes = align_up((size_t)s.batch * s.h_q * window * 4, 256);
   bd_shape ls = s;
@@ -1275,7 +1342,7 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
     p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
     p.seq_lens = s.seq_lens;
     p.h_kv = s.h_kv;
-    void* fn = score_fn(s.head_dim, plan.nq_pad).fn;
+    void* fn = score_fn(s.head_dim, plan.nq_pad, s.seq_lens != nullptr).fn;
     err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
     if (err != cudaSuccess) return err;
     void* args[] = {&p, &kmap, &qmap};

@@ -50,18 +50,37 @@ struct VerifyParams {
 
 // The global tile list is cut into equal CTA ranges after every unit's tiles are preceded
 // by `seg_cost` virtual tiles: a CTA whose range starts a unit (and so stops to merge one
-// segment and load new queries) receives that many fewer real tiles.  Virtual index v of
-// unit u = v / (tpu + a) maps to the unit's first real tile while inside its virtual prefix.
-__host__ __device__ __forceinline__ int real_tile(int v, int tpu, int a) {
-  const int u = v / (tpu + a);
-  const int r = v - u * (tpu + a);
-  return u * tpu + (r > a ? r - a : 0);
-}
+// segment and load new queries) receives that many fewer real tiles.
 // The CTA whose range holds real tile g.
 __host__ __device__ __forceinline__ int tile_owner(int g, int tpu, int a, int vtpc) {
   const int u = g / tpu;
   return (u * (tpu + a) + a + (g - u * tpu)) / vtpc;
 }
+
+// The same layout seen per unit: unit u spans virtual tiles [vbase(u), vbase(u + 1)), its
+// `a` virtual tiles first, then its real tiles 0 .. tiles(u) - 1; the list is cut into
+// ranges of vtpc virtual tiles, one per CTA.  pref (shared memory, per-sequence lengths)
+// holds vbase(u) for u = 0 .. units; null means every unit has tpu real tiles.
+struct VerifyMap {
+  const int* pref;
+  int tpu, a, units, vtpc;
+  __device__ __forceinline__ int vbase(int u) const { return pref ? pref[u] : u * (tpu + a); }
+  __device__ __forceinline__ int tiles(int u) const { return vbase(u + 1) - vbase(u) - a; }
+  __device__ __forceinline__ int unit_of(int v) const {   // the unit whose span holds v
+    if (!pref) return v / (tpu + a);
+    int lo = 0, hi = units - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (pref[mid] <= v) lo = mid;
+      else hi = mid - 1;
+    }
+    return lo;
+  }
+  // real tiles of unit u inside the virtual range [v0, v1)
+  __device__ __forceinline__ int first_tile(int u, int v0) const { return max(0, v0 - vbase(u) - a); }
+  __device__ __forceinline__ int end_tile(int u, int v1) const { return min(tiles(u), v1 - vbase(u) - a); }
+  __device__ __forceinline__ int owner(int u, int tile) const { return (vbase(u) + a + tile) / vtpc; }
+};
 
 template <int D, int NT, int WQ, bool WITH_V>
 struct VerifySmem {
@@ -85,13 +104,6 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   constexpr uint32_t HALF_BYTES = kVKeys * 128;
   constexpr int STAGES = kVStages;
 
-  const int n_units = p.total_tiles / p.tiles_per_unit;
-  const int v_end = n_units * (p.tiles_per_unit + p.seg_cost);
-  const int g0 = real_tile(blockIdx.x * p.vtiles_per_cta, p.tiles_per_unit, p.seg_cost);
-  const int g1 = real_tile(min((blockIdx.x + 1) * p.vtiles_per_cta, v_end), p.tiles_per_unit, p.seg_cost);
-  if (g0 >= g1) return;                           // whole CTA idle
-  const int ntiles = g1 - g0;
-
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem);
@@ -104,8 +116,47 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   float* f_s = l_s + WK * NQC;
   float* o_s = f_s + WK * NQC;
   float* w_s = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(m_s) + L::kMerge);
+  int* pref = reinterpret_cast<int*>(reinterpret_cast<uint8_t*>(w_s) + L::kWeights);   // ragged: [units + 1]
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int n_units = p.total_tiles / p.tiles_per_unit;
+  VerifyMap map{nullptr, p.tiles_per_unit, p.seg_cost, n_units, p.vtiles_per_cta};
+  if (p.seq_lens) {
+    // per-sequence lengths: every CTA lays out the units' virtual tile spans itself (the
+    // lengths may come from the preceding kernel, so after the dependency wait)
+    grid_dependency_wait();
+    int* wtot = reinterpret_cast<int*>(smem + 512);
+    const int per = (n_units + kVThreads - 1) / kVThreads;
+    const int u0 = min(n_units, tid * per), u1 = min(n_units, u0 + per);
+    auto span = [&](int u) {
+      const int t_u = max(0, unit_context(p.seq_lens, u, p.h_kv, p.t_ctx - p.len_offset, nullptr) + p.len_offset);
+      return (t_u + p.n_q + kVKeys - 1) / kVKeys + p.seg_cost;
+    };
+    int sum = 0;
+    for (int u = u0; u < u1; ++u) sum += span(u);
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    if (lane == 31) wtot[warp] = incl;
+    __syncthreads();
+    int run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += wtot[w];
+    for (int u = u0; u < u1; ++u) {
+      pref[u] = run;
+      run += span(u);
+    }
+    if (tid == kVThreads - 1) pref[n_units] = run;
+    __syncthreads();
+    map.pref = pref;
+    map.vtpc = max((pref[n_units] + (int)gridDim.x - 1) / (int)gridDim.x, p.vtiles_per_cta);
+  }
+  const int v_total = map.vbase(n_units);
+  const int v0 = min(v_total, (int)blockIdx.x * map.vtpc), v1 = min(v_total, v0 + map.vtpc);
+  if (v0 >= v1) return;                           // whole CTA idle
+  const int u_first = map.unit_of(v0), u_last = map.unit_of(v1 - 1);
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
       mbar_init(&full_bar[s], 1);
@@ -124,32 +175,34 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
       if (WITH_V) tma_prefetch_map(&vmap);
       int issued = 0;
       // with per-sequence lengths any tile may hold some sequence's block rows (written by
-      // the preceding kernels): wait before the first load
-      bool waited = false;
-      if (p.seq_lens) {
-        grid_dependency_wait();
-        waited = true;
-      }
-      for (int t = 0; t < ntiles; ++t) {
-        const int s = t % STAGES;
-        if (t >= STAGES && !mbar_wait(&empty_bar[s], ((t / STAGES) & 1) ^ 1, p.status, abort_flag)) break;
-        const int g = g0 + t;
-        const int unit = g / p.tiles_per_unit;
-        const int key0 = (g % p.tiles_per_unit) * kVKeys;
-        if (!waited && key0 + kVKeys > p.t_ctx) {      // this tile holds rows of the block itself
-          grid_dependency_wait();
-          waited = true;
-        }
-        uint8_t* st = stage_base + s * L::STAGE_BYTES;
-        mbar_arrive_expect_tx(&full_bar[s], L::STAGE_BYTES);
+      // the preceding kernels): the wait above came before the first load
+      bool waited = p.seq_lens != nullptr;
+      bool stop = false;
+      for (int unit = u_first; unit <= u_last && !stop; ++unit) {
+        const int tb = map.first_tile(unit, v0), te = map.end_tile(unit, v1);
+        for (int tile = tb; tile < te; ++tile) {
+          const int t = issued;
+          const int s = t % STAGES;
+          if (t >= STAGES && !mbar_wait(&empty_bar[s], ((t / STAGES) & 1) ^ 1, p.status, abort_flag)) {
+            stop = true;
+            break;
+          }
+          const int key0 = tile * kVKeys;
+          if (!waited && key0 + kVKeys > p.t_ctx) {    // this tile holds rows of the block itself
+            grid_dependency_wait();
+            waited = true;
+          }
+          uint8_t* st = stage_base + s * L::STAGE_BYTES;
+          mbar_arrive_expect_tx(&full_bar[s], L::STAGE_BYTES);
 #pragma unroll
-        for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * HALF_BYTES, &kmap, &full_bar[s], 64 * h, key0, unit);
-        if (WITH_V) {
+          for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * HALF_BYTES, &kmap, &full_bar[s], 64 * h, key0, unit);
+          if (WITH_V) {
 #pragma unroll
-          for (int h = 0; h < D / 64; ++h)
-            tma_load_3d(st + L::TILE_BYTES + h * HALF_BYTES, &vmap, &full_bar[s], 64 * h, key0, unit);
+            for (int h = 0; h < D / 64; ++h)
+              tma_load_3d(st + L::TILE_BYTES + h * HALF_BYTES, &vmap, &full_bar[s], 64 * h, key0, unit);
+          }
+          issued = t + 1;
         }
-        issued = t + 1;
       }
       if (*abort_flag) {   // never leave a copy in flight behind an aborted CTA
         for (int t = max(0, issued - STAGES); t < issued; ++t)
@@ -170,9 +223,9 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
 
   bool alive = true;   // false once this warp's wait gave up (the abort flag is then set)
   int t = 0;
-  for (int seg_start = g0; seg_start < g1;) {
-    const int unit = seg_start / p.tiles_per_unit;
-    const int seg_end = min(g1, (unit + 1) * p.tiles_per_unit);
+  for (int unit = u_first; unit <= u_last; ++unit) {
+    const int tb = map.first_tile(unit, v0), te = map.end_tile(unit, v1);
+    if (tb >= te) continue;                      // only virtual tiles of this unit here
     const int t_unit = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx - p.len_offset, tid == 0 ? p.status : nullptr) +
                        p.len_offset;
 #pragma unroll
@@ -186,7 +239,7 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     WarpAttn<D, NT, WITH_V>::load_q(bq, p.q + (size_t)unit * nq * D, nq, wq * NT, lane);
     WarpAttn<D, NT, WITH_V> wa;
     wa.init();
-    for (int g = seg_start; g < seg_end && alive; ++g, ++t) {
+    for (int tile = tb; tile < te && alive; ++tile, ++t) {
       const int s = t % STAGES;
       if (!mbar_wait(&full_bar[s], (t / STAGES) & 1, p.status, abort_flag)) {
         alive = false;
@@ -194,7 +247,7 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
       }
       const uint32_t kbase = smem_u32(stage_base + s * L::STAGE_BYTES);
       const uint32_t vbase = kbase + L::TILE_BYTES;
-      const int key_tile0 = (g % p.tiles_per_unit) * kVKeys;
+      const int key_tile0 = tile * kVKeys;
 #pragma unroll
       for (int sub = 0; sub < SUBS; ++sub) {
         const int kb = 16 * (wk + WK * sub);
@@ -211,8 +264,8 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     wa.store(m_s, l_s, o_s, wk, NQC, wq * NT, lane);
     named_bar(1, NCT);
     const int c = blockIdx.x;
-    const int c_first = tile_owner(unit * p.tiles_per_unit, p.tiles_per_unit, p.seg_cost, p.vtiles_per_cta);
-    const int c_last = tile_owner((unit + 1) * p.tiles_per_unit - 1, p.tiles_per_unit, p.seg_cost, p.vtiles_per_cta);
+    const int c_first = map.owner(unit, 0);
+    const int c_last = map.owner(unit, map.tiles(unit) - 1);
     const int n_seg = c_last - c_first + 1;
     const size_t row0 = (size_t)unit * nq;
     if (n_seg == 1) {
@@ -241,7 +294,6 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     if (tid == 0) last_flag[1] = *abort_flag;
     named_bar(1, NCT);
     if (last_flag[1]) break;
-    seg_start = seg_end;
   }
 }
 
@@ -348,6 +400,15 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   }
   if (max_seg > kVMaxSeg) return false;
   plan->max_seg = max_seg;
+  if (s.seq_lens) {
+    // per-sequence lengths: the kernel cuts the ranges itself over the actual tiles, no
+    // shorter than the bound that keeps every unit within kVMaxSeg segments; the units'
+    // span table takes (units + 1) ints of shared memory
+    plan->tiles_per_cta = (int)((tpu + a + kVMaxSeg - 2) / (kVMaxSeg - 1));
+    plan->max_seg = kVMaxSeg;
+    plan->smem_bytes += align_up((size_t)(units + 1) * 4, 16);
+    if (plan->smem_bytes > 227 * 1024) return false;
+  }
   return true;
 }
 
@@ -392,10 +453,10 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.max_seg = plan.max_seg;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const KernelInfo k = select_kernel(s.head_dim, plan.nt, plan.wq, plan.with_v);
-  err = cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)k.smem);
+  err = cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
   if (err != cudaSuccess) return err;
   void* args[] = {&p, &kmap, &vmap};
-  return launch_kernel(k.fn, dim3(plan.grid), dim3(kVThreads), k.smem, stream, args, 0);
+  return launch_kernel(k.fn, dim3(plan.grid), dim3(kVThreads), plan.smem_bytes, stream, args, 0);
 }
 
 }  // namespace bd
