@@ -288,6 +288,17 @@ int bd_write_block_rows(const bd_shape* shape, int n_rows, const void* k_rows, c
                         void* v_cache, void* stream);
 
 /*
+ * Diagnostic of the device-side error path (the paper has no counterpart): launches one
+ * small kernel that waits on a shared-memory barrier nothing completes, gives up after
+ * limit_us microseconds (1 .. 2000000) like every bounded wait in the library, records
+ * BD_ERR_TIMEOUT in the workspace's status word and returns; a second warp waiting on the
+ * same barrier stops through the shared abort flag, as the roles of a pipelined kernel do.
+ * No fault, trap or hang: the context stays usable, and bd_workspace_status() then reads
+ * BD_ERR_TIMEOUT.  ws needs only the 256-byte status header.
+ */
+int bd_check_wait_timeout(void* ws, size_t ws_bytes, int limit_us, void* stream);
+
+/*
  * Reads (and clears) the device status word of a workspace: BD_OK, or the first
  * device-side error recorded by a kernel since the last read.  Synchronises
  * `stream`.  Returns BD_ERR_INVALID_ARG for a NULL ws, BD_ERR_CUDA if the copy fails.

@@ -20,6 +20,7 @@ from .binding import (  # noqa: F401
     bd_accept,
     bd_advance,
     bd_argmax,
+    bd_check_wait_timeout,
     bd_combine,
     bd_draft_attn,
     bd_draft_attn_static,

@@ -54,6 +54,7 @@ _SIGNATURES = {
     "bd_advance": (ctypes.c_int, [_SHAPE, ctypes.c_int, ctypes.c_int, _P, _P, _P, _P, _P, _P, _P, ctypes.c_int, _P,
                                   _P]),
     "bd_write_block_rows": (ctypes.c_int, [_SHAPE, ctypes.c_int, _P, _P, _P, _P, _P]),
+    "bd_check_wait_timeout": (ctypes.c_int, [_P, ctypes.c_size_t, ctypes.c_int, _P]),
     "bd_workspace_status": (ctypes.c_int, [_P, _P]),
     "bd_strerror": (ctypes.c_char_p, [ctypes.c_int]),
 }
@@ -220,6 +221,12 @@ def bd_write_block_rows(shape, n_rows, k_rows, v_rows, k_cache, v_cache, stream=
     st = library().bd_write_block_rows(ctypes.byref(shape), int(n_rows), _ptr(k_rows), _ptr(v_rows), _ptr(k_cache),
                                        _ptr(v_cache), _stream(stream))
     _check("bd_write_block_rows", st)
+
+
+def bd_check_wait_timeout(ws: Workspace, limit_us: int, stream=None):
+    """Runs the bounded-wait error path once (see the header); read the result with
+    bd_workspace_status."""
+    _check("bd_check_wait_timeout", library().bd_check_wait_timeout(ws.ptr, ws.nbytes, int(limit_us), _stream(stream)))
 
 
 def bd_workspace_status(ws: Workspace, stream=None) -> int:

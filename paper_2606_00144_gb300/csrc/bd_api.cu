@@ -357,6 +357,14 @@ int bd_write_block_rows(const bd_shape* shape, int n_rows, const void* k_rows, c
   return BD_OK;
 }
 
+int bd_check_wait_timeout(void* ws, size_t ws_bytes, int limit_us, void* stream) {
+  if (!ws) return BD_ERR_INVALID_ARG;
+  if (ws_bytes < kWsHeaderBytes) return BD_ERR_WORKSPACE;
+  if (limit_us < 1 || limit_us > 2000000) return BD_ERR_INVALID_ARG;
+  BD_TRY(check_tensor(ws, 16));
+  return map_cuda(launch_wait_probe(status_word(ws), limit_us, static_cast<cudaStream_t>(stream)));
+}
+
 int bd_workspace_status(void* ws, void* stream) {
   if (!ws) return BD_ERR_INVALID_ARG;
   int host = 0;

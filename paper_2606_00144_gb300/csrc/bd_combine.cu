@@ -39,4 +39,32 @@ cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_spl
   return launch_kernel(fn, grid, dim3(kCThreads), smem, stream, args, 0);
 }
 
+// The error path of a bounded wait, end to end: one warp waits on a shared-memory barrier
+// that nothing completes until limit_ns runs out, which records BD_ERR_TIMEOUT in the status
+// word exactly as a stalled pipeline wait of the other kernels does, and the kernel returns.
+// The second warp watches the shared abort flag the waiting warp raises and stops too.
+__global__ void __launch_bounds__(64) wait_probe_kernel(int* status, unsigned long long limit_ns) {
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    mbar_fence_init();
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    if (threadIdx.x == 0) mbar_wait_for(&bar, 0, status, &abort_flag, limit_ns);
+  } else if (threadIdx.x == 32) {
+    // a second role that gives up once the first has: the abort flag ends its wait
+    mbar_wait_for(&bar, 0, nullptr, &abort_flag, 4 * limit_ns);
+  }
+  __syncthreads();
+}
+
+cudaError_t launch_wait_probe(int* status, long long limit_us, cudaStream_t stream) {
+  unsigned long long ns = (unsigned long long)limit_us * 1000ull;
+  void* args[] = {&status, &ns};
+  return launch_kernel(reinterpret_cast<void*>(&wait_probe_kernel), dim3(1), dim3(64), 0, stream, args, 0);
+}
+
 }  // namespace bd

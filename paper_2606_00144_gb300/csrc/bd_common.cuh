@@ -122,8 +122,8 @@ __device__ __forceinline__ bool mbar_test(uint32_t addr, uint32_t parity) {
 // Bounded wait for the completion of the barrier phase with the given parity.
 // `abort_flag` (shared) lets one timed-out role stop the others quickly.  Returns false
 // on timeout or abort; the caller then skips its remaining work.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status,
-                                          volatile int* abort_flag) {
+__device__ __forceinline__ bool mbar_wait_for(uint64_t* bar, uint32_t parity, int* status,
+                                              volatile int* abort_flag, uint64_t limit_ns) {
   const uint32_t addr = smem_u32(bar);
   if (mbar_test(addr, parity)) return true;
   const uint64_t t0 = global_timer_ns();
@@ -131,12 +131,16 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
     if (mbar_test(addr, parity)) return true;
     if ((i & 31u) == 31u) {
       if (abort_flag && *abort_flag) return false;
-      if (global_timer_ns() - t0 > kWaitLimitNs) break;
+      if (global_timer_ns() - t0 > limit_ns) break;
     }
   }
   record_error(status, BD_ERR_TIMEOUT);
   if (abort_flag) *abort_flag = 1;
   return false;
+}
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* status,
+                                          volatile int* abort_flag) {
+  return mbar_wait_for(bar, parity, status, abort_flag, kWaitLimitNs);
 }
 
 // ---------------------------------------------------------------------------------------

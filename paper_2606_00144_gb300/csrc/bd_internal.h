@@ -94,6 +94,7 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_split, int rows,
                            int head_dim, void* o_out, float* lse_out, cudaStream_t stream);
 int combine_rows_per_block(int n_split);
+cudaError_t launch_wait_probe(int* status, long long limit_us, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------- acceptance
 int argmax_cluster(int rows, int vocab);   // CTAs per row

@@ -201,3 +201,12 @@ def test_plain_c_consumer(lib, tmp_path):
     assert out[2] == f"argmax {INVALID}"
     assert out[3] == f"accept_empty {BD_OK}"
     assert out[4] == "strerror " + bd.bd_strerror(MISALIGNED)
+
+
+def test_check_wait_timeout_validation(lib):
+    f = lib.bd_check_wait_timeout
+    assert f(None, 1024, 1000, None) == INVALID
+    assert f(A, 16, 1000, None) == WORKSPACE
+    assert f(A, 1024, 0, None) == INVALID
+    assert f(A, 1024, 3000000, None) == INVALID
+    assert f(A + 4, 1024, 1000, None) == MISALIGNED
