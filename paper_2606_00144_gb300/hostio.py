@@ -104,46 +104,63 @@ class HostStepIO:
     def run(self, n_steps):
         """Issues n_steps pipelined steps on the current stream (capturable in a CUDA graph).
 
-        Step s: its packed queries are copied once the kernels of step s-2 (the slot's last
-        reader) are done, and its K/V rows once step s-1's kernels are done; its selection
-        waits for the queries and for the result copy of step s-2 (the slot's last writer),
-        its draft passes for the rows; its results are copied once its kernels are done."""
+        Step s+1's packed queries are copied during step s, once step s-1's kernels (the
+        slot's last readers) are done; step s+1's K/V rows once step s's kernels are done;
+        step s's results once its kernels are done.  Every wait of the compute stream on
+        a copy sits just before a step's first draft pass, so the selection and verify
+        kernels keep their programmatic (overlapping) launches: before step s's first draft
+        pass it waits for its rows, for step s+1's queries and for step s-1's result copy
+        (the last reader of the slot step s+1 writes)."""
+        if n_steps < 1:
+            return
         cs = torch.cuda.current_stream()
         xi, xo = self.in_stream, self.out_stream
         xi.wait_stream(cs)
         xo.wait_stream(cs)
         L = range(len(self.layers))
-        done = [None, None]      # kernels of the last step that used the slot
-        drained = [None, None]   # result copy of the last step that used the slot
-        prev = None              # kernels of the previous step
-        for s in range(n_steps):
-            slot = s % 2
+        g = self.layers[0][0].gamma
+
+        def copy_queries(step):
+            e = torch.cuda.Event()
             with torch.cuda.stream(xi):
-                if done[slot] is not None:
-                    xi.wait_event(done[slot])
-                self.d_in[slot].copy_(self.h_in[slot], non_blocking=True)
-                q_ready = torch.cuda.Event()
-                q_ready.record(xi)
-                if prev is not None:
-                    xi.wait_event(prev)
-                hr = self.prow.views(self.h_rows[slot])
+                self.d_in[step % 2].copy_(self.h_in[step % 2], non_blocking=True)
+                e.record(xi)
+            return e
+
+        def copy_rows(step):
+            e = torch.cuda.Event()
+            with torch.cuda.stream(xi):
+                hr = self.prow.views(self.h_rows[step % 2])
                 for l in L:
                     st, k_cache, v_cache, _ = self.layers[l]
                     B.bd_write_block_rows(st.shape, st.gamma + 1, hr[f"k_rows{l}"], hr[f"v_rows{l}"], k_cache,
                                           v_cache, xi)
-                rows_ready = torch.cuda.Event()
-                rows_ready.record(xi)
+                e.record(xi)
+            return e
+
+        q_ready = copy_queries(0)
+        rows_ready = copy_rows(0)
+        cs.wait_event(q_ready)
+        done = [None] * n_steps
+        drained = [None] * n_steps
+        for s in range(n_steps):
+            slot = s % 2
+            if s + 1 < n_steps:
+                if s >= 1:
+                    xi.wait_event(done[s - 1])
+                q_next = copy_queries(s + 1)
             vin = self.pin.views(self.d_in[slot])
             vout = self.pout.views(self.d_out[slot])
-            cs.wait_event(q_ready)
-            if drained[slot] is not None:
-                cs.wait_event(drained[slot])
             for l in L:
                 st, k_cache, _, carry = self.layers[l]
                 self._bind(l, vout)
                 st.select(k_cache, vin[f"q_win{l}"], vin[f"lse{l}"] if carry else None)
             cs.wait_event(rows_ready)
-            for j in range(self.layers[0][0].gamma):
+            if s + 1 < n_steps:
+                cs.wait_event(q_next)
+            if s >= 1:
+                cs.wait_event(drained[s - 1])
+            for j in range(g):
                 for l in L:
                     st, k_cache, v_cache, _ = self.layers[l]
                     self._bind(l, vout)
@@ -152,13 +169,15 @@ class HostStepIO:
                 st, k_cache, v_cache, _ = self.layers[l]
                 self._bind(l, vout)
                 st.verify(vin[f"q_verify{l}"], k_cache, v_cache)
-            done[slot] = torch.cuda.Event()
-            done[slot].record(cs)
-            prev = done[slot]
+            done[s] = torch.cuda.Event()
+            done[s].record(cs)
+            if s + 1 < n_steps:
+                xi.wait_event(done[s])
+                rows_ready = copy_rows(s + 1)
             with torch.cuda.stream(xo):
-                xo.wait_event(done[slot])
+                xo.wait_event(done[s])
                 self.h_out[slot].copy_(self.d_out[slot], non_blocking=True)
-                drained[slot] = torch.cuda.Event()
-                drained[slot].record(xo)
+                drained[s] = torch.cuda.Event()
+                drained[s].record(xo)
         cs.wait_stream(xi)
         cs.wait_stream(xo)
