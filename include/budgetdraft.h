@@ -74,7 +74,8 @@ typedef enum bd_status {
  * advanced on the device by bd_advance); t_ctx is then the longest length and sizes the
  * launches.  Everything this header says of t_ctx holds per sequence with T_b in its
  * place.  NULL: every sequence has t_ctx.  A T_b outside [1, t_ctx] is recorded in the
- * workspace status word (BD_ERR_INVALID_ARG) and clamped into range. */
+ * workspace status word (BD_ERR_INVALID_ARG) and clamped into range.  With seq_lens,
+ * batch * h_kv must not exceed 1024 (BD_ERR_UNSUPPORTED). */
 typedef struct bd_shape {
   int32_t batch;     /* sequences                                   */
   int32_t h_q;       /* query heads                                 */

@@ -105,6 +105,8 @@ int check_shape(const bd_shape* s) {
   // every per-unit row offset must stay addressable by the TMA (rows < 2^31)
   if ((long long)s->batch * s->h_kv * s->t_cap >= (1LL << 31)) return BD_ERR_UNSUPPORTED;
   if (s->seq_lens && !aligned(s->seq_lens, 4)) return BD_ERR_MISALIGNED;
+  // per-sequence lengths: the kernels keep a per-unit table in shared memory
+  if (s->seq_lens && (long long)s->batch * s->h_kv > kMaxRaggedUnits) return BD_ERR_UNSUPPORTED;
   return BD_OK;
 }
 

@@ -210,3 +210,9 @@ def test_check_wait_timeout_validation(lib):
     assert f(A, 1024, 0, None) == INVALID
     assert f(A, 1024, 3000000, None) == INVALID
     assert f(A + 4, 1024, 1000, None) == MISALIGNED
+
+
+def test_seq_lens_unit_limit(lib):
+    s = shape(batch=129, h_q=64, h_kv=8)          # 1032 units
+    s.seq_lens = A
+    assert verify(lib, s) == UNSUPPORTED
