@@ -11,10 +11,10 @@ can check each function against the paper by eye.
 
 Paper references (BudgetDraft, arXiv 2606.00144):
   * Sparse drafter view K_S^sp(B) selected from the drafter prefix cache under a
-    KV budget B: Sec. 3.1 (Eq. p_S) and the TopKChunks construction in Sec. 3.4
-    ("partition the prefix cache into chunks, score each chunk by cumulative
-    attention weight, keep the top floor(B/s) chunks"), used by Algorithm 1
-    step 4 and by the sparsify line of Algorithm 2.
+    KV budget B: Sec. 3.1 (Eq. p_S) and the TopKChunks construction of Sec. 3.4
+    (the prefix is cut into chunks of s positions, each chunk is ranked by the
+    attention weight it accumulates, and the best floor(B/s) chunks are kept), which
+    Algorithm 1 and the sparsify step of Algorithm 2 both use.
   * Draft step: gamma autoregressive drafter steps over K_S^sp(B) (Algorithm 2,
     Draft; Sec. 3.5).
   * Verify step: the verifier checks all gamma drafts in one forward over the
