@@ -20,6 +20,9 @@
  *   bd_write_block_rows  writes the block's new K/V rows into the caches;
  *   bd_advance        slides the observation window over the settled block rows and
  *                     appends their positions to the sparse view (Algorithm 2, Update).
+ * Around them: bd_workspace_size / bd_workspace_status (scratch and device-side
+ * errors), bd_draft_attn_static (bd_draft_attn without a workspace),
+ * bd_check_wait_timeout (runs the device-side error path on purpose) and bd_strerror.
  *
  * Conventions shared by every call
  *   - All tensor arguments are DEVICE pointers owned by the caller (the row sources
