@@ -129,7 +129,8 @@ size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q);
  *               NULL to have it computed here (reads K a second time).
  *   idx_out     int32 [batch, h_kv, budget]: kept positions ascending, then -1 padding.
  *   count_out   int32 [batch, h_kv]: number of kept positions.
- * Constraints: 1 <= window <= t_ctx, (h_q/h_kv)*window <= 256, n_sink, n_recent >= 0,
+ * Constraints: 1 <= window <= t_ctx, (h_q/h_kv)*window <= 256 (<= 128 with window_lse
+ * NULL: the LSE pass runs on the lse-only verify kernel), n_sink, n_recent >= 0,
  * n_sink + n_recent <= budget when budget < t_ctx, chunk >= 1, t_cap >= t_ctx.
  */
 int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_window,

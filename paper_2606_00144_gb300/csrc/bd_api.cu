@@ -185,6 +185,7 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
   if ((s.h_q / s.h_kv) * window > 256) return BD_ERR_UNSUPPORTED;
   SelectPlan sp;
   if (!select_plan(s, window, budget, n_sink, n_recent, chunk, &sp)) return BD_ERR_UNSUPPORTED;
+  if (!window_lse && sp.need_scores && !sp.self_mode) return BD_ERR_UNSUPPORTED;   // > 128 window rows per KV head
   if (!ws) return BD_ERR_WORKSPACE;
   if (!aligned(ws, 256)) return BD_ERR_MISALIGNED;
   const int units = s.batch * s.h_kv;

@@ -81,6 +81,7 @@ struct SelectPlan {
   size_t smem_bytes;
   size_t score_bytes, lse_bytes;
   VerifyPlan lse_plan;  // self mode: window LSE through the verify kernel (lse only)
+  bool self_mode;       // lse_plan is valid (the window rows fit the lse-only kernel)
 };
 bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_recent, int chunk,
                  SelectPlan* plan);

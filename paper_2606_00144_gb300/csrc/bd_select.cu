@@ -1288,13 +1288,15 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   plan->lse_bytes = align_up((size_t)s.batch * s.h_q * window * 4, 256);
   bd_shape ls = s;
   ls.t_ctx = s.t_ctx - window;
-  if (!verify_plan(ls, window, false, &plan->lse_plan)) return false;
+  // self mode runs the window LSE through the lse-only verify kernel (at most 128 query
+  // rows per KV head); carry mode does not need it
+  plan->self_mode = verify_plan(ls, window, false, &plan->lse_plan);
   return true;
 }
 
 size_t select_region_bytes(const bd_shape& s, const SelectPlan& plan) {
   bd_shape ls = s;
-  return plan.score_bytes + plan.lse_bytes + verify_partials_bytes(ls, plan.lse_plan);
+  return plan.score_bytes + (plan.self_mode ? plan.lse_bytes + verify_partials_bytes(ls, plan.lse_plan) : 0);
 }
 
 cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void* k_cache,

@@ -100,6 +100,7 @@ def test_select_validation(lib):
     assert select(lib, shape(), sink=-1) == INVALID
     assert select(lib, shape(), lse=A + 1) == MISALIGNED
     assert select(lib, shape(h_q=16, h_kv=1), window=32) == UNSUPPORTED  # 512 window rows > 256
+    assert select(lib, shape(h_q=16, h_kv=2), window=32, lse=None) == UNSUPPORTED   # self mode: 256 rows > 128
     assert select(lib, shape(), qw=0) == INVALID
 
 

@@ -197,6 +197,8 @@ RAGGED = [
     (1, 8, 2, 128, 1031, 128, 4, 32, 32, 5, 8),   # chunks with sink/recent and ragged chunk edges
     (1, 8, 2, 128, 300, 36, 4, 32, 32, 1, 1),     # B = sink + recent: nothing ranked
     (1, 8, 2, 64, 40, 64, 4, 8, 32, 5, 1),        # B > T
+    (1, 16, 2, 128, 700, 100, 4, 16, 32, 2, 1),   # group 8 x window 32 = 256 rows: two TMEM accumulators, one Q buffer
+    (2, 16, 2, 64, 900, 120, 4, 16, 32, 2, 1),    # the same at d 64
     (1, 8, 2, 128, 20000, 600, 4, 64, 32, 1, 1),  # 16K < middle <= 32K: the shared-memory top-B kernel
     (1, 4, 1, 64, 40000, 300, 4, 32, 32, 1, 1),   # middle > 32K: the general top-B kernel
 ]
@@ -208,7 +210,8 @@ def test_ragged_shapes(case):
     wl = W.tiny_workload(batch=b, h_q=hq, h_kv=hkv, head_dim=d, t_ctx=t, budget=budget, n_sink=sink,
                          n_recent=recent, window=window, gamma=gamma, seed=11 + t)
     inp = W.make_layer(wl, 0, "cuda")
-    run_and_check(wl, inp, host(inp), chunk=chunk, tag=f"ragged{case}")
+    modes = ("carry", "self") if (hq // hkv) * window <= 128 else ("carry",)   # self mode: <= 128 window rows
+    run_and_check(wl, inp, host(inp), chunk=chunk, tag=f"ragged{case}", modes=modes)
 
 
 @pytest.mark.parametrize("n_q,with_v", [(1, True), (2, True), (12, True), (21, True), (32, False)])
