@@ -131,7 +131,8 @@ class Workspace:
         sizes = [bd_workspace_size(shape, BD_OP_SELECT, budget, window),
                  bd_workspace_size(shape, BD_OP_DRAFT, budget, gamma),
                  bd_workspace_size(shape, BD_OP_VERIFY, budget, gamma + 1)]
-        if min(sizes) == 0:
+        # an op this shape does not support reports size 0 here and its status when called
+        if max(sizes) == 0:
             raise BudgetDraftError("bd_workspace_size", -1)
         return cls(max(sizes), device)
 
