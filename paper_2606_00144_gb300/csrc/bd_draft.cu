@@ -37,13 +37,14 @@ constexpr int kDThreads = 32 * kDWarps;
 constexpr int kDMaxCluster = 8;   // CTAs per (sequence, KV head): the portable cluster size
 
 struct DraftParams {
-  const __nv_bfloat16* q;      // [units * G][D]
+  const __nv_bfloat16* q;      // [units * g][D]
   const __nv_bfloat16* k;      // [units][t_cap][D]
   const __nv_bfloat16* v;
   const int32_t* idx;          // [units][budget]
   const int32_t* count;        // [units]
-  __nv_bfloat16* o;            // [units * G][D]
-  float* lse;                  // [units * G] or null
+  __nv_bfloat16* o;            // [units * g][D]
+  float* lse;                  // [units * g] or null
+  int g;                       // query heads of a KV head (<= the kernel's G; the rest are padding)
   int* status;
   const int32_t* seq_lens;      // per-sequence context lengths [batch] or null (all t_ctx)
   int h_kv;
@@ -165,7 +166,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     if (n_tiles > 0) gather(0, 0, 1);
   }
   uint32_t bq[1][D / 16][2];
-  WarpAttn<D, 1, true>::load_q(bq, p.q + (size_t)unit * G * D, G, 0, lane);
+  WarpAttn<D, 1, true>::load_q(bq, p.q + (size_t)unit * p.g * D, p.g, 0, lane);
   WarpAttn<D, 1, true> wa;
   wa.init();
   for (int t = 0; t < n_tiles; ++t) {
@@ -199,9 +200,9 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   wa.finish_rows();
   wa.store(m_s, l_s, o_s, warp, 8, 0, lane);
   __syncthreads();
-  const size_t row0 = (size_t)unit * G;
+  const size_t row0 = (size_t)unit * p.g;
   if (p.n_split == 1) {
-    merge_warps_and_store<D, kDWarps, true>(m_s, l_s, f_s, o_s, 8, G, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D,
+    merge_warps_and_store<D, kDWarps, true>(m_s, l_s, f_s, o_s, 8, p.g, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D,
                                             true, tid, kDThreads, 0);
     return;
   }
@@ -215,7 +216,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   cluster.sync();                                  // all partials have landed in rank 0
   if (rank != 0) return;
   float* wts = o_s;                                // [C][G] merge weights
-  if (tid < G) {
+  if (tid < p.g) {
     float mx = -INFINITY;
     for (int r = 0; r < C; ++r) mx = fmaxf(mx, parts[r * (G * D + G) + G * D + tid]);
     float tot = 0.f;
@@ -230,7 +231,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     if (p.lse) p.lse[row0 + tid] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
   }
   __syncthreads();
-  for (int i = tid; i < G * (D / 2); i += kDThreads) {
+  for (int i = tid; i < p.g * (D / 2); i += kDThreads) {
     const int g = i / (D / 2), d = (i % (D / 2)) * 2;
     float a0 = 0.f, a1 = 0.f;
     for (int r = 0; r < C; ++r) {
@@ -265,9 +266,12 @@ size_t smem_bytes(int d, int g, int n_stage, int cluster) {
 }
 }  // namespace
 
+// The kernel instance whose n8 query tile holds a group of g query heads (g <= 8).
+int draft_group_instance(int g) { return g <= 1 ? 1 : g <= 2 ? 2 : g <= 4 ? 4 : 8; }
+
 bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
   const int g = s.h_q / s.h_kv;
-  if (!pick(s.head_dim, g)) return false;
+  if (g < 1 || g > 8 || !pick(s.head_dim, draft_group_instance(g))) return false;
   const long entries = (long)budget + n_steps;
   int n_split = (int)std::min<long>((entries + kDRows - 1) / kDRows, kDMaxCluster);
   n_split = std::max(n_split, 1);
@@ -307,8 +311,10 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.flags = flags;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const int g = s.h_q / s.h_kv;
-  void* fn = pick(s.head_dim, g);
-  const size_t smem = smem_bytes(s.head_dim, g, p.n_stage, plan.n_split);
+  const int g_kernel = draft_group_instance(g);
+  p.g = g;
+  void* fn = pick(s.head_dim, g_kernel);
+  const size_t smem = smem_bytes(s.head_dim, g_kernel, p.n_stage, plan.n_split);
   cudaError_t err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
 
