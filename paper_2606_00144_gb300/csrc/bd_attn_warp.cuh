@@ -222,4 +222,53 @@ __device__ __forceinline__ void merge_warps_and_store(const float* m_s, const fl
   }
 }
 
+// One-pass form of merge_warps_and_store for the draft pass: each thread owns four
+// adjacent output columns of one row and derives that row's merge factors itself from
+// the WK warps' (m, l) (broadcast shared-memory loads), so no barrier separates the
+// factors from the output.  o_dst rows are D wide (bf16 if OUT_BF16 else fp32, written
+// 8 or 16 bytes at a time: o_dst must be 16-byte aligned); lse_dst[r] in natural log.
+template <int D, int WK, bool OUT_BF16>
+__device__ __forceinline__ void merge_warps_flat(const float* m_s, const float* l_s, const float* o_s, int nqc,
+                                                 int n_cols, float* lse_dst, void* o_dst, int tid, int n_threads) {
+  constexpr int OP = D + 4;
+  constexpr int Q = D / 4;
+  for (int i = tid; i < n_cols * Q; i += n_threads) {
+    const int col = i / Q, d = (i % Q) * 4;
+    float mw[WK];
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < WK; ++w) {
+      mw[w] = m_s[w * nqc + col];
+      M = fmaxf(M, mw[w]);
+    }
+    const float M_use = M == -INFINITY ? 0.f : M;
+    float L = 0.f;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int w = 0; w < WK; ++w) {
+      const float f = fast_exp2(mw[w] - M_use);
+      L += f * l_s[w * nqc + col];
+      const float4 v = *reinterpret_cast<const float4*>(o_s + (size_t)(w * nqc + col) * OP + d);
+      a.x += f * v.x;
+      a.y += f * v.y;
+      a.z += f * v.z;
+      a.w += f * v.w;
+    }
+    const float inv = L > 0.f ? 1.f / L : 0.f;
+    a.x *= inv;
+    a.y *= inv;
+    a.z *= inv;
+    a.w *= inv;
+    if (d == 0 && lse_dst) lse_dst[col] = L > 0.f ? (M + log2f(L)) * kLn2 : -INFINITY;
+    if (OUT_BF16) {
+      uint2 packed;
+      packed.x = pack_bf16x2(a.x, a.y);
+      packed.y = pack_bf16x2(a.z, a.w);
+      *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(o_dst) + (size_t)col * D + d) = packed;
+    } else {
+      *reinterpret_cast<float4*>(static_cast<float*>(o_dst) + (size_t)col * D + d) = a;
+    }
+  }
+}
+
 }  // namespace bd

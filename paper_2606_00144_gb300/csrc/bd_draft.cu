@@ -59,11 +59,13 @@ struct DraftSmem {
   static constexpr uint32_t TILE_BYTES = kDRows * D * 2;
   static constexpr uint32_t STAGE_BYTES = 2 * TILE_BYTES;                 // K and V
   static constexpr size_t kMerge = (size_t)(3 * kDWarps * 8) * 4 + (size_t)kDWarps * 8 * (D + 4) * 4;
+  // one CTA's partial in rank 0: G rows of D floats, then G lse padded to 16 bytes
+  static constexpr int kSlot = G * D + ((G + 3) & ~3);
   // stages (the warp-merge scratch reuses them) | rowpos [2][kDRows] |
-  // partials of the cluster's CTAs [C][G*D + G] (used in rank 0 only)
+  // partials of the cluster's CTAs [C][kSlot] (used in rank 0 only)
   static size_t bytes(int n_stage, int cluster) {
     const size_t stages = std::max<size_t>((size_t)n_stage * STAGE_BYTES, kMerge);
-    return 1024 + stages + 2 * kDRows * 4 + (size_t)cluster * (G * D + G) * 4 + 16;
+    return 1024 + stages + 2 * kDRows * 4 + (size_t)cluster * kSlot * 4 + 16;
   }
 };
 
@@ -85,7 +87,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
                                                                                : kMergeBytes;
   uint8_t* stage = smem;                                                  // n_stage x (K, V)
   int* rowpos = reinterpret_cast<int*>(smem + stage_bytes);               // [2][kDRows]
-  float* parts = reinterpret_cast<float*>(rowpos + 2 * kDRows);           // [C][G*D + G]
+  float* parts = reinterpret_cast<float*>(rowpos + 2 * kDRows);           // [C][kSlot]
   float* m_s = reinterpret_cast<float*>(stage);                           // warp-merge scratch
   float* l_s = m_s + kDWarps * 8;
   float* f_s = l_s + kDWarps * 8;
@@ -202,45 +204,50 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   __syncthreads();
   const size_t row0 = (size_t)unit * p.g;
   if (p.n_split == 1) {
-    merge_warps_and_store<D, kDWarps, true>(m_s, l_s, f_s, o_s, 8, p.g, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D,
-                                            true, tid, kDThreads, 0);
+    merge_warps_flat<D, kDWarps, true>(m_s, l_s, o_s, 8, p.g, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D, tid,
+                                       kDThreads);
     return;
   }
   // ---------------------------------------------------------------- cluster merge (DSMEM)
+  constexpr int SLOT = L::kSlot;
   cg::cluster_group cluster = cg::this_cluster();
   const int C = p.n_split;
   const int rank = (int)cluster.block_rank();
-  float* slot = cluster.map_shared_rank(parts, 0) + (size_t)rank * (G * D + G);   // in rank 0
+  float* slot = cluster.map_shared_rank(parts, 0) + (size_t)rank * SLOT;   // in rank 0
   asm volatile("barrier.cluster.wait.aligned;" ::: "memory");          // every CTA is running
-  merge_warps_and_store<D, kDWarps, true>(m_s, l_s, f_s, o_s, 8, G, slot + G * D, slot, false, tid, kDThreads, 0);
+  merge_warps_flat<D, kDWarps, false>(m_s, l_s, o_s, 8, G, slot + G * D, slot, tid, kDThreads);
   cluster.sync();                                  // all partials have landed in rank 0
   if (rank != 0) return;
-  float* wts = o_s;                                // [C][G] merge weights
-  if (tid < p.g) {
+  // each thread: four output columns of one head, its merge weights derived in place
+  for (int i = tid; i < p.g * (D / 4); i += kDThreads) {
+    const int g = i / (D / 4), d = (i % (D / 4)) * 4;
+    float lr[kDMaxCluster];
     float mx = -INFINITY;
-    for (int r = 0; r < C; ++r) mx = fmaxf(mx, parts[r * (G * D + G) + G * D + tid]);
+#pragma unroll
+    for (int r = 0; r < kDMaxCluster; ++r) {
+      lr[r] = r < C ? parts[r * SLOT + G * D + g] : -INFINITY;
+      mx = fmaxf(mx, lr[r]);
+    }
     float tot = 0.f;
-    for (int r = 0; r < C; ++r) {
-      const float l = parts[r * (G * D + G) + G * D + tid];
-      const float w = mx == -INFINITY ? 0.f : fast_exp2((l - mx) * kLog2e);
-      wts[r * G + tid] = w;
-      tot += w;
+    float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int r = 0; r < kDMaxCluster; ++r) {
+      if (r < C) {
+        const float w = mx == -INFINITY ? 0.f : fast_exp2((lr[r] - mx) * kLog2e);
+        const float4 v = *reinterpret_cast<const float4*>(parts + r * SLOT + g * D + d);
+        tot += w;
+        a.x += w * v.x;
+        a.y += w * v.y;
+        a.z += w * v.z;
+        a.w += w * v.w;
+      }
     }
     const float inv = tot > 0.f ? 1.f / tot : 0.f;
-    for (int r = 0; r < C; ++r) wts[r * G + tid] *= inv;
-    if (p.lse) p.lse[row0 + tid] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
-  }
-  __syncthreads();
-  for (int i = tid; i < p.g * (D / 2); i += kDThreads) {
-    const int g = i / (D / 2), d = (i % (D / 2)) * 2;
-    float a0 = 0.f, a1 = 0.f;
-    for (int r = 0; r < C; ++r) {
-      const float w = wts[r * G + g];
-      const float2 v = *reinterpret_cast<const float2*>(parts + r * (G * D + G) + g * D + d);
-      a0 += w * v.x;
-      a1 += w * v.y;
-    }
-    *reinterpret_cast<uint32_t*>(p.o + (row0 + g) * D + d) = pack_bf16x2(a0, a1);
+    uint2 packed;
+    packed.x = pack_bf16x2(a.x * inv, a.y * inv);
+    packed.y = pack_bf16x2(a.z * inv, a.w * inv);
+    *reinterpret_cast<uint2*>(p.o + (row0 + g) * D + d) = packed;
+    if (d == 0 && p.lse) p.lse[row0 + g] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
   }
 }
 
