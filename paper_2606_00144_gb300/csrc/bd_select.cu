@@ -986,7 +986,9 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
   const float* sc = p.score + (size_t)unit * p.n_mid_pad;
   const int w0 = warp * ROWS * 32;
 
-  // ---- the thread's scores (fp32 bits; non-negative, so their order is the bits' order)
+  // ---- the thread's scores (fp32 bits; non-negative, so their order is the bits' order).
+  // Slots past n hold +0: no score is below it and ties go to the lower position, so the
+  // padding never displaces a real score and needs no test in the passes below.
   uint32_t u[ROWS];
   float lmin = INFINITY, lmax = -INFINITY;
 #pragma unroll
@@ -994,10 +996,8 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     const int i = w0 + 32 * r + lane;
     const float v = i < n ? __ldcg(sc + i) : 0.f;
     u[r] = __float_as_uint(v);
-    if (i < n) {
-      lmin = fminf(lmin, v);
-      lmax = fmaxf(lmax, v);
-    }
+    lmin = fminf(lmin, v);
+    lmax = fmaxf(lmax, v);
   }
   for (int i = tid; i < kBins; i += kTopkThreads) bins[i] = 0;
 #pragma unroll
@@ -1015,11 +1015,11 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     s_eq_all = 0;
   }
   __syncthreads();
-  float vmin = wmin[0], vmax = wmax[0];
-#pragma unroll 8
-  for (int w = 1; w < 32; ++w) {
-    vmin = fminf(vmin, wmin[w]);
-    vmax = fmaxf(vmax, wmax[w]);
+  float vmin = wmin[lane], vmax = wmax[lane];
+#pragma unroll
+  for (int off = 16; off > 0; off >>= 1) {
+    vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, off));
+    vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, off));
   }
 
   // ---- tau (bits of the k-th largest score) and krem (how many scores equal to tau to keep)
@@ -1029,8 +1029,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     const float scale = (float)(kBins - 1) / (vmax - vmin);
     auto bin_of = [&](uint32_t x) -> int { return min(kBins - 1, (int)((__uint_as_float(x) - vmin) * scale)); };
 #pragma unroll
-    for (int r = 0; r < ROWS; ++r)
-      if (w0 + 32 * r + lane < n) atomicAdd(&bins[bin_of(u[r])], 1u);
+    for (int r = 0; r < ROWS; ++r) atomicAdd(&bins[bin_of(u[r])], 1u);
     __syncthreads();
     constexpr int BPT = kBins / kTopkThreads;
     uint32_t hb[BPT];
@@ -1076,7 +1075,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
 #pragma unroll
       for (int r = 0; r < ROWS; ++r) {
         const int i = w0 + 32 * r + lane;
-        if (i < n && bin_of(u[r]) == bstar)
+        if (bin_of(u[r]) == bstar)
           cand[atomicAdd(&s_nc, 1u)] = (static_cast<uint64_t>(u[r]) << 32) | (0xFFFFFFFFu - (uint32_t)i);
       }
       __syncthreads();
@@ -1113,7 +1112,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
       __syncthreads();
 #pragma unroll
       for (int r = 0; r < ROWS; ++r)
-        if (w0 + 32 * r + lane < n && (u[r] & mask) == prefix) atomicAdd(&bins[(u[r] >> shift) & 255u], 1u);
+        if ((u[r] & mask) == prefix) atomicAdd(&bins[(u[r] >> shift) & 255u], 1u);
       __syncthreads();
       if (warp == 0) {
         uint32_t local = 0;
@@ -1155,7 +1154,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     uint32_t eqc = 0;
 #pragma unroll
     for (int r = 0; r < ROWS; ++r)
-      eqc += __popc(__ballot_sync(0xffffffffu, w0 + 32 * r + lane < n && u[r] == tau));
+      eqc += __popc(__ballot_sync(0xffffffffu, u[r] == tau));
     if (lane == 0) wsum[warp] = eqc;
     __syncthreads();
     if (warp == 0) {
@@ -1176,9 +1175,8 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
   uint32_t cnt = 0, eq_run = eq_base;
 #pragma unroll
   for (int r = 0; r < ROWS; ++r) {
-    const bool valid = w0 + 32 * r + lane < n;
-    bool sel = valid && u[r] > tau;
-    const bool eq = valid && u[r] == tau;
+    bool sel = u[r] > tau;
+    const bool eq = u[r] == tau;
     if (simple) {
       sel |= eq;
     } else {

@@ -339,6 +339,24 @@ def test_tied_scores_take_lowest_positions(planted):
     run_and_check(wl, inp, host(inp), check_steps=False, tag=f"ties planted={planted}")
 
 
+def test_boundary_among_underflowed_scores():
+    """Window queries along one axis and middle keys pointing the other way: their scores
+    underflow to exactly 0 in fp32 (the oracle's fp64 values are ~1e-150, inside the tie
+    band), only every 100th key scores above 0, so the budget boundary falls among the
+    zeros.  The top-B then has to take real zero-score positions in position order ahead
+    of the zero padding of its register rows (5964 middle scores in 8192 slots)."""
+    wl = W.tiny_workload(batch=1, h_q=8, h_kv=2, head_dim=128, t_ctx=6000, budget=300, n_sink=4, n_recent=32,
+                         window=32, gamma=1)
+    inp = W.make_layer(wl, 0, "cuda")
+    inp.q_win.mul_(0.05)
+    inp.q_win[..., 0] = 64.0
+    mid = inp.k_cache[:, :, wl.n_sink: wl.t_ctx - wl.n_recent]
+    mid.mul_(0.05)
+    mid[..., 0] = -64.0
+    mid[:, :, ::100, 0] = 64.0
+    run_and_check(wl, inp, host(inp), check_steps=False, tag="boundary among zero scores")
+
+
 def test_determinism():
     wl = W.WORKLOADS["l8b_4k"]
     inp = W.make_layer(wl, 0, "cuda")
