@@ -445,6 +445,28 @@ def extras(step, args):
                      "GB/s": round(lb / (us_acc * 1e-6) / 1e9, 1), "launches_per_step": wl.gamma + 2,
                      "step_with_accept_us": round(us_full, 2)}
 
+    # self mode: the window LSE computed in the call instead of carried (same inputs)
+    if step.budget < wl.t_ctx and step.sel_mode == "carry":
+        v = Step(wl, step.budget, step.n_recent, "self", "cuda", share=step)
+        v.lse = [None] * wl.layers
+        us = time_per_step(v.run, n, gs)
+        pb = step_bytes(wl, step.budget, step.n_recent, "self")["total"] * wl.layers
+        out["self_mode"] = {"us_per_step": round(us, 2), "GB/s": round(pb / (us * 1e-6) / 1e9, 1),
+                            "bytes_per_step": pb, "launches_per_step": v.launches_per_step()}
+        del v
+
+    # token-level budget sweep with a recent window of B/4 (B >= T keeps the whole context)
+    rows = []
+    for bb in (256, 512, 1024, 2048, wl.t_ctx):
+        rec = min(bb // 4, wl.t_ctx)
+        v = Step(wl, bb, rec, step.sel_mode, "cuda", share=step)
+        us = time_per_step(v.run, n, gs)
+        pb = step_bytes(wl, bb, rec, step.sel_mode)["total"] * wl.layers
+        rows.append({"budget": bb, "n_recent": rec, "us_per_step": round(us, 2),
+                     "GB/s": round(pb / (us * 1e-6) / 1e9, 1), "bytes_per_step": pb})
+        del v
+    out["budget_sweep"] = rows
+
     # the paper's chunk policy (Sec. 3.4, s = 8): same sink/recent/budget, and the pure
     # top-floor(B/s)-chunks form with no sink or recent window over a budget sweep
     if step.budget < wl.t_ctx:

@@ -50,6 +50,7 @@ struct DraftParams {
   int h_kv;
   int budget, step_j, t_ctx, t_cap, n_split, rows_per_split;
   int n_stage;                 // 1, or 2 when a CTA gathers more than one tile (double buffer)
+  int pos_slots;               // rows_per_split rounded up to whole tiles (row positions in shared memory)
   unsigned flags;              // BD_DRAFT_VIEW_READY: gather the selected rows before the dependency wait
   float scale_log2;
 };
@@ -61,11 +62,11 @@ struct DraftSmem {
   static constexpr size_t kMerge = (size_t)(3 * kDWarps * 8) * 4 + (size_t)kDWarps * 8 * (D + 4) * 4;
   // one CTA's partial in rank 0: G rows of D floats, then G lse padded to 16 bytes
   static constexpr int kSlot = G * D + ((G + 3) & ~3);
-  // stages (the warp-merge scratch reuses them) | rowpos [2][kDRows] |
-  // partials of the cluster's CTAs [C][kSlot] (used in rank 0 only)
-  static size_t bytes(int n_stage, int cluster) {
+  // stages (the warp-merge scratch reuses them) | rowpos [pos_slots] (the row of every
+  // entry of the CTA's slice) | partials of the cluster's CTAs [C][kSlot] (rank 0 only)
+  static size_t bytes(int n_stage, int cluster, int pos_slots) {
     const size_t stages = std::max<size_t>((size_t)n_stage * STAGE_BYTES, kMerge);
-    return 1024 + stages + 2 * kDRows * 4 + (size_t)cluster * kSlot * 4 + 16;
+    return 1024 + stages + (size_t)pos_slots * 4 + (size_t)cluster * kSlot * 4 + 16;
   }
 };
 
@@ -86,8 +87,8 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   const size_t stage_bytes = (size_t)p.n_stage * L::STAGE_BYTES > kMergeBytes ? (size_t)p.n_stage * L::STAGE_BYTES
                                                                                : kMergeBytes;
   uint8_t* stage = smem;                                                  // n_stage x (K, V)
-  int* rowpos = reinterpret_cast<int*>(smem + stage_bytes);               // [2][kDRows]
-  float* parts = reinterpret_cast<float*>(rowpos + 2 * kDRows);           // [C][kSlot]
+  int* rowpos = reinterpret_cast<int*>(smem + stage_bytes);               // [pos_slots]
+  float* parts = reinterpret_cast<float*>(rowpos + p.pos_slots);          // [C][kSlot]
   float* m_s = reinterpret_cast<float*>(stage);                           // warp-merge scratch
   float* l_s = m_s + kDWarps * 8;
   float* f_s = l_s + kDWarps * 8;
@@ -127,15 +128,15 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     }
     return idx_value;
   };
-  // row positions of tile `tile` into rowpos[b] (threads < kDRows), then the gather
-  auto set_rows = [&](int tile, int b, bool prefetched) {
-    const int e0 = e_begin + tile * kDRows;
+  // the row of every entry of the slice, up front: tile 0 from the prefetched indices, the
+  // later tiles' loads all in flight together (no index round trip between tiles)
+  auto set_all_rows = [&]() {
     if (tid < kDRows) {
-      const int e = e0 + tid;
-      int pos = -1;
-      if (e < e_end) pos = position(e, prefetched ? idx_pref : (e < cnt ? __ldg(iunit + e) : 0));
-      rowpos[b * kDRows + tid] = pos;
+      const int e = e_begin + tid;
+      rowpos[tid] = e < e_end ? position(e, idx_pref) : -1;
     }
+    for (int e = e_begin + kDRows + tid; e < e_end; e += kDThreads)
+      rowpos[e - e_begin] = position(e, e < cnt ? __ldg(iunit + e) : 0);
   };
   // part 0: context rows (and zero fill), part 1: drafted rows (t_ctx and later), part 2: all
   auto gather = [&](int tile, int b, int part) {
@@ -144,12 +145,12 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     uint8_t* vt = kt + L::TILE_BYTES;
     for (int c = tid; c < kDRows * CH; c += kDThreads) {
       const int r = c / CH, ch = c % CH;
-      const int pos = rowpos[b * kDRows + r];
+      const int pos = rowpos[tile * kDRows + r];
       const bool live = r < nrows && pos >= 0;   // others zero-filled (0 * garbage could be NaN in P V)
       const bool drafted = live && pos >= t_unit;
       if ((part == 0 && drafted) || (part == 1 && !drafted)) continue;
       const uint32_t off = sw128_offset(r, ch * 8, HALF_BYTES);
-      const size_t src = (size_t)max(pos, 0) * D + ch * 8;
+      const size_t src = live ? (size_t)pos * D + ch * 8 : 0;   // slots past the slice are not initialised
       cp_async16_zfill(kt + off, kunit + src, live);
       cp_async16_zfill(vt + off, vunit + src, live);
     }
@@ -158,7 +159,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
 
   const bool dbuf = p.n_stage == 2;
   if (n_tiles > 0) {
-    set_rows(0, 0, true);
+    set_all_rows();
     __syncthreads();
     gather(0, 0, early ? 0 : 2);
   }
@@ -174,8 +175,6 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   for (int t = 0; t < n_tiles; ++t) {
     const int b = dbuf ? (t & 1) : 0;
     if (dbuf && t + 1 < n_tiles) {
-      set_rows(t + 1, (t + 1) & 1, false);
-      __syncthreads();
       gather(t + 1, (t + 1) & 1, 2);
       cp_async_wait<1>();
     } else {
@@ -184,7 +183,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     __syncthreads();
     const int nrows = min(kDRows, e_end - (e_begin + t * kDRows));
     const uint32_t kbase = smem_u32(stage + b * L::STAGE_BYTES);
-    const int* rp = rowpos + b * kDRows;
+    const int* rp = rowpos + t * kDRows;
     if (16 * warp < nrows) {
       const int kb = 16 * warp;
       wa.step(kbase, kbase + L::TILE_BYTES, HALF_BYTES, kb, bq, p.scale_log2, lane, [&](int ko, int, int) {
@@ -193,11 +192,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
       });
     }
     __syncthreads();                              // buffer b is free again
-    if (!dbuf && t + 1 < n_tiles) {
-      set_rows(t + 1, 0, false);
-      __syncthreads();
-      gather(t + 1, 0, 2);
-    }
+    if (!dbuf && t + 1 < n_tiles) gather(t + 1, 0, 2);
   }
   wa.finish_rows();
   wa.store(m_s, l_s, o_s, warp, 8, 0, lane);
@@ -263,9 +258,9 @@ DraftFn pick(int d, int g) {
 #undef BD_DK
   return nullptr;
 }
-size_t smem_bytes(int d, int g, int n_stage, int cluster) {
+size_t smem_bytes(int d, int g, int n_stage, int cluster, int pos_slots) {
 #define BD_DS(DD, GG) \
-  if (d == DD && g == GG) return DraftSmem<DD, GG>::bytes(n_stage, cluster);
+  if (d == DD && g == GG) return DraftSmem<DD, GG>::bytes(n_stage, cluster, pos_slots);
   BD_DS(64, 1) BD_DS(64, 2) BD_DS(64, 4) BD_DS(64, 8)
   BD_DS(128, 1) BD_DS(128, 2) BD_DS(128, 4) BD_DS(128, 8)
 #undef BD_DS
@@ -280,7 +275,12 @@ bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
   const int g = s.h_q / s.h_kv;
   if (g < 1 || g > 8 || !pick(s.head_dim, draft_group_instance(g))) return false;
   const long entries = (long)budget + n_steps;
+  // one tile per CTA up to a cluster of 8, but no more CTAs than one wave holds (about three
+  // single-stage CTAs per SM): a second wave would repeat the whole latency chain of a pass
+  const long units = (long)s.batch * s.h_kv;
+  const long wave = 3L * current_sm_count();
   int n_split = (int)std::min<long>((entries + kDRows - 1) / kDRows, kDMaxCluster);
+  n_split = (int)std::min<long>(n_split, std::max<long>(1, wave / std::max<long>(1, units)));
   n_split = std::max(n_split, 1);
   plan->n_entries_max = (int)entries;
   plan->rows_per_split = (int)((entries + n_split - 1) / n_split);
@@ -314,14 +314,23 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.t_cap = s.t_cap;
   p.n_split = plan.n_split;
   p.rows_per_split = plan.rows_per_split;
-  p.n_stage = plan.rows_per_split > kDRows ? 2 : 1;
+  // double buffering (twice the tile memory, two CTAs per SM) where the grid still fits one
+  // wave at that occupancy, or where a CTA walks three tiles or more (a long loop gains more
+  // from overlapping its own gathers than from a single wave); a CTA of two tiles in a
+  // larger grid relies on its co-resident CTAs to hide its gathers
+  p.n_stage = (plan.rows_per_split > kDRows && (long)units * plan.n_split <= 2L * current_sm_count()) ||
+                      plan.rows_per_split > 2 * kDRows
+                  ? 2
+                  : 1;
+  p.pos_slots = (plan.rows_per_split + kDRows - 1) / kDRows * kDRows;
   p.flags = flags;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const int g = s.h_q / s.h_kv;
   const int g_kernel = draft_group_instance(g);
   p.g = g;
   void* fn = pick(s.head_dim, g_kernel);
-  const size_t smem = smem_bytes(s.head_dim, g_kernel, p.n_stage, plan.n_split);
+  const size_t smem = smem_bytes(s.head_dim, g_kernel, p.n_stage, plan.n_split, p.pos_slots);
+  if (smem > 227 * 1024) return cudaErrorInvalidValue;
   cudaError_t err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (err != cudaSuccess) return err;
 

@@ -18,11 +18,13 @@ from tests.parity import check_attention, f64
 pytestmark = pytest.mark.gpu
 
 
-def test_draft_attn_static_matches_workspace_entry_point():
+@pytest.mark.parametrize("budget", [512, 2048])
+def test_draft_attn_static_matches_workspace_entry_point(budget):
+    """budget 2048: every CTA of a unit's cluster gathers several tiles."""
     bd.build()
     wl = W.WORKLOADS["l8b_16k_b8"]
     inp = W.make_layer(wl, 0, "cuda")
-    st = bd.SpecStep.for_workload(wl)
+    st = bd.SpecStep.for_workload(wl, budget=budget, n_recent=budget // 4)
     st.select(inp.k_cache, inp.q_win, None)                 # a real sparse view to gather
     o = torch.empty(wl.batch, wl.h_q, wl.head_dim, dtype=torch.bfloat16, device="cuda")
     lse = torch.empty(wl.batch, wl.h_q, device="cuda")
@@ -31,7 +33,7 @@ def test_draft_attn_static_matches_workspace_entry_point():
         bd.bd_draft_attn_static(st.shape, inp.q_draft[j], inp.k_cache, inp.v_cache, st.idx, st.count,
                                 st.budget, j, o, lse)
         torch.cuda.synchronize()
-        check_attention(o, lse, f64(st.draft_o[j]), f64(st.draft_lse[j]), f"static draft j={j}")
+        check_attention(o, lse, f64(st.draft_o[j]), f64(st.draft_lse[j]), f"static draft B={budget} j={j}")
     assert st.ws.status() == 0
 
 
