@@ -214,8 +214,10 @@ class Step:
         if marks:
             record(marks[0])
         if select:
+            # the window queries and LSE are this step's inputs, written before the kernel
+            # that precedes the selection (the previous step's verify)
             for l in L:
-                self.steps[l].select(self.layers[l].k_cache, self.layers[l].q_win, self.lse[l])
+                self.steps[l].select(self.layers[l].k_cache, self.layers[l].q_win, self.lse[l], window_ready=True)
         if marks:
             record(marks[1])
         for j in range(self.wl.gamma):

@@ -105,6 +105,14 @@ enum { BD_OP_SELECT = 1, BD_OP_DRAFT = 2, BD_OP_VERIFY = 3 };
  */
 size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q);
 
+/* bd_select_budget flags. */
+enum {
+  /* q_window (and window_lse) were written before the kernel that immediately precedes
+   * this call on `stream` (not by it: bd_advance, for one, rewrites them in place): the
+   * call may load the window queries while that kernel finishes. */
+  BD_SELECT_WINDOW_READY = 1
+};
+
 /*
  * KV-budget selection: the sparse drafter view K_S^sp(B) of every (sequence, KV
  * head).  Sec. 3.4 of the paper keeps the top floor(B/s) chunks of the prefix by
@@ -127,16 +135,17 @@ size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q);
  *   window_lse  fp32 [batch, h_q, window]: each window row's softmax normaliser over
  *               keys [0, p_w] (carried from the step that verified that token), or
  *               NULL to have it computed here (reads K a second time).
+ *   flags       0 or BD_SELECT_WINDOW_READY.
  *   idx_out     int32 [batch, h_kv, budget]: kept positions ascending, then -1 padding.
  *   count_out   int32 [batch, h_kv]: number of kept positions.
  * Constraints: 1 <= window <= t_ctx, (h_q/h_kv)*window <= 256 (<= 128 with window_lse
- * NULL: the LSE pass runs on the lse-only verify kernel), n_sink, n_recent >= 0,
+ * NULL), n_sink, n_recent >= 0,
  * n_sink + n_recent <= budget when budget < t_ctx, chunk >= 1, t_cap >= t_ctx.
  */
 int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_window,
                      const float* window_lse, int window, int budget, int n_sink, int n_recent,
-                     int chunk, int32_t* idx_out, int32_t* count_out, void* ws, size_t ws_bytes,
-                     void* stream);
+                     int chunk, unsigned flags, int32_t* idx_out, int32_t* count_out, void* ws,
+                     size_t ws_bytes, void* stream);
 
 /* bd_draft_attn flags. */
 enum {

@@ -9,6 +9,7 @@ seeded synthetic workloads.
 
 from .binding import (  # noqa: F401
     BD_DRAFT_VIEW_READY,
+    BD_SELECT_WINDOW_READY,
     BD_DTYPE_BF16,
     BD_DTYPE_F32,
     BD_OP_DRAFT,

@@ -17,6 +17,7 @@ from .build import LIB_PATH
 BD_OK = 0
 BD_OP_SELECT, BD_OP_DRAFT, BD_OP_VERIFY = 1, 2, 3
 BD_DRAFT_VIEW_READY = 1
+BD_SELECT_WINDOW_READY = 1
 BD_DTYPE_BF16, BD_DTYPE_F32 = 1, 2
 
 
@@ -42,7 +43,8 @@ _SHAPE = ctypes.POINTER(BdShape)
 _SIGNATURES = {
     "bd_workspace_size": (ctypes.c_size_t, [_SHAPE, ctypes.c_int, ctypes.c_int, ctypes.c_int]),
     "bd_select_budget": (ctypes.c_int, [_SHAPE, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int,
-                                        ctypes.c_int, ctypes.c_int, _P, _P, _P, ctypes.c_size_t, _P]),
+                                        ctypes.c_int, ctypes.c_int, ctypes.c_uint, _P, _P, _P, ctypes.c_size_t,
+                                        _P]),
     "bd_draft_attn": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_uint, _P,
                                      _P, _P, ctypes.c_size_t, _P]),
     "bd_draft_attn_static": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P,
@@ -145,10 +147,11 @@ class Workspace:
 
 
 def bd_select_budget(shape, k_cache, q_window, window_lse, window, budget, n_sink, n_recent, chunk,
-                     idx_out, count_out, ws: Workspace, stream=None):
+                     idx_out, count_out, ws: Workspace, stream=None, flags=0):
     st = library().bd_select_budget(ctypes.byref(shape), _ptr(k_cache), _ptr(q_window), _ptr(window_lse),
                                     int(window), int(budget), int(n_sink), int(n_recent), int(chunk),
-                                    _ptr(idx_out), _ptr(count_out), ws.ptr, ws.nbytes, _stream(stream))
+                                    int(flags), _ptr(idx_out), _ptr(count_out), ws.ptr, ws.nbytes,
+                                    _stream(stream))
     _check("bd_select_budget", st)
 
 

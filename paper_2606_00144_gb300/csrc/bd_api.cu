@@ -170,7 +170,7 @@ size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q) {
 }
 
 int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_window, const float* window_lse,
-                     int window, int budget, int n_sink, int n_recent, int chunk, int32_t* idx_out,
+                     int window, int budget, int n_sink, int n_recent, int chunk, unsigned flags, int32_t* idx_out,
                      int32_t* count_out, void* ws, size_t ws_bytes, void* stream) {
   BD_TRY(check_shape(shape));
   const bd_shape& s = *shape;
@@ -182,6 +182,7 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
   if (window < 1 || window > s.t_ctx || budget < 1 || n_sink < 0 || n_recent < 0 || chunk < 1)
     return BD_ERR_INVALID_ARG;
   if (budget < s.t_ctx && n_sink + n_recent > budget) return BD_ERR_INVALID_ARG;
+  if (flags & ~BD_SELECT_WINDOW_READY) return BD_ERR_INVALID_ARG;
   if ((s.h_q / s.h_kv) * window > 256) return BD_ERR_UNSUPPORTED;
   SelectPlan sp;
   if (!select_plan(s, window, budget, n_sink, n_recent, chunk, &sp)) return BD_ERR_UNSUPPORTED;
@@ -191,7 +192,7 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
   const int units = s.batch * s.h_kv;
   if (ws_bytes < ws_region_offset(units) + select_region_bytes(s, sp)) return BD_ERR_WORKSPACE;
   return map_cuda(launch_select(s, sp, k_cache, q_window, window_lse, window, budget, n_sink, n_recent, chunk,
-                                idx_out, count_out, region(ws, units), counters(ws), status_word(ws),
+                                flags, idx_out, count_out, region(ws, units), counters(ws), status_word(ws),
                                 static_cast<cudaStream_t>(stream)));
 }
 

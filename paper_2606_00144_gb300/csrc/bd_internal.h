@@ -81,14 +81,17 @@ struct SelectPlan {
   size_t smem_bytes;
   size_t score_bytes, lse_bytes;
   VerifyPlan lse_plan;  // self mode: window LSE through the verify kernel (lse only)
-  bool self_mode;       // lse_plan is valid (the window rows fit the lse-only kernel)
+  bool self_mode;       // the window LSE can be computed here (one of the two kernels below)
+  bool lse_tc;          // self mode on window_lse_kernel (tcgen05) rather than the verify kernel
+  int lse_tiles_per_unit, lse_total_tiles, lse_tiles_per_cta, lse_grid, lse_max_seg;
+  size_t lse_smem_bytes, lse_part_bytes;
 };
 bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_recent, int chunk,
                  SelectPlan* plan);
 size_t select_region_bytes(const bd_shape& s, const SelectPlan& plan);
 cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void* k_cache,
                           const void* q_window, const float* window_lse, int window, int budget,
-                          int n_sink, int n_recent, int chunk, int32_t* idx_out, int32_t* count_out,
+                          int n_sink, int n_recent, int chunk, unsigned flags, int32_t* idx_out, int32_t* count_out,
                           void* ws_region, int* counters, int* status, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------- combine

@@ -7,8 +7,9 @@
 //               row: no cross-thread reduction.  Persistent CTAs (one per SM):
 //                 warp 0   producer: K tiles by TMA (128-byte swizzle, 4-stage ring) and the
 //                          unit's window queries into a double-buffered swizzled Q tile;
-//                          both are context data, streamed before the grid-dependency
-//                          wait, which only the epilogue (reading the window LSE) takes;
+//                          the first stages' K tiles (context rows) stream before the
+//                          grid-dependency wait, the queries (which bd_advance may have
+//                          just rewritten) and the later tiles after it;
 //                 warp 1   one lane issues tcgen05.mma into four fp32 TMEM accumulators
 //                          (two when the window rows need more columns) and commits to
 //                          the smem/TMEM barriers;
@@ -51,6 +52,7 @@ struct ScoreParams {
   float scale_log2;
   const int32_t* seq_lens;      // per-sequence context lengths [batch] or null (all t_ctx)
   int h_kv;
+  int window_ready;             // BD_SELECT_WINDOW_READY: the queries may load before the dependency wait
 };
 
 // RAGGED: per-sequence lengths (the tile layout is built on the device); a separate
@@ -170,6 +172,33 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
       tma_prefetch_map(&kmap);
       tma_prefetch_map(&qmap);
     }
+    // K tile i into its ring stage (lane 0; false once a wait gave up)
+    int k_issued = 0;
+    auto issue_k = [&](int i) -> bool {
+      bool ok = true;
+      if (lane == 0) {
+        int unit, tt;
+        locate(first + i, unit, tt);
+        const int s = i % STAGES;
+        if (i >= STAGES) ok = mbar_wait(&empty_bar[s], ((i / STAGES) & 1) ^ 1, p.status, abort_flag);
+        if (ok) {
+          uint8_t* st = kstage + s * KTILE;
+          mbar_arrive_expect_tx(&full_bar[s], KTILE);
+          const int key0 = p.n_sink + kSKeys * tt;
+#pragma unroll
+          for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * KHALF, &kmap, &full_bar[s], 64 * h, key0, unit);
+          k_issued = i + 1;
+        }
+      }
+      return __shfl_sync(0xffffffffu, ok, 0);
+    };
+    // the first stages' K tiles (context rows, which the kernel just before never writes)
+    // stream before the grid-dependency wait; the window queries may come from that kernel
+    // (bd_advance rewrites them in place), so they load after it, unless the caller says
+    // they were written earlier (then queries and tiles interleave from the start)
+    const int pre = p.window_ready ? 0 : min(n, STAGES);
+    for (int i = 0; i < pre; ++i) issue_k(i);
+    if (!p.window_ready) grid_dependency_wait();
     int cur_unit = -1, qcount = 0;
     for (int i = 0; i < n; ++i) {
       const int g = first + i;
@@ -194,19 +223,13 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
         cur_unit = unit;
         ++qcount;
       }
-      bool ok = true;
-      if (lane == 0) {
-        const int s = i % STAGES;
-        if (i >= STAGES) ok = mbar_wait(&empty_bar[s], ((i / STAGES) & 1) ^ 1, p.status, abort_flag);
-        if (ok) {
-          uint8_t* st = kstage + s * KTILE;
-          mbar_arrive_expect_tx(&full_bar[s], KTILE);
-          const int key0 = p.n_sink + kSKeys * tt;
-#pragma unroll
-          for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * KHALF, &kmap, &full_bar[s], 64 * h, key0, unit);
-        }
-      }
-      if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+      if (i >= pre && !issue_k(i)) break;
+    }
+    if (lane == 0 && *abort_flag) {   // no copy may land in shared memory after the CTA exits
+      for (int t = max(0, k_issued - STAGES); t < k_issued; ++t)
+        mbar_wait(&full_bar[t % STAGES], (t / STAGES) & 1, p.status, nullptr);
+      for (int q = max(0, qcount - NQB); q < qcount; ++q)
+        mbar_wait(&qfull_bar[q % NQB], (q / NQB) & 1, p.status, nullptr);
     }
   } else if (warp == 1) {
     // ---------------------------------------------------------------- MMA issuer
@@ -338,6 +361,277 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
   __syncthreads();
   tc_fence_after();
   if (warp == 1) tmem_dealloc(tmem_base, p.tmem_cols);
+}
+
+// ============================================================================ window LSE
+//
+// Self mode's normalisers: lse_r = log sum_{k <= p_w} exp(q_r . k_k / sqrt(d)) for the G*W
+// window rows r = h*W + w of every unit (p_w = t_ctx - W + w).  The contraction of
+// score_kernel with its operands swapped: the unit's window rows are the A operand (M =
+// 128 rows = the TMEM lanes) and a 128-key K tile the B operand (N = 128 columns), so each
+// of the four epilogue warps' threads owns one window row and keeps that row's online
+// log-sum-exp in registers, with no cross-thread reduction.  Persistent CTAs (one per SM)
+// take contiguous ranges of the (unit, 128-key tile) list: warp 0 streams K tiles (TMA,
+// 4-stage ring) and the unit's rows (two buffers), warp 1 issues the MMAs into four TMEM
+// accumulators, warps 2-5 reduce.  A unit split over several CTAs merges the segments'
+// (max, sum) pairs in the CTA that finishes it last.
+struct LseParams {
+  float* lse;          // [units * nq_rows] natural log
+  float2* part;        // [units][max_seg][128]: a segment's (running max in log2 units, sum)
+  int* counters;       // [units] arrival counters (left zero)
+  int* status;
+  int nq_rows, window, t_ctx, tiles_per_unit, total_tiles, tiles_per_cta, max_seg;
+  int window_ready;    // BD_SELECT_WINDOW_READY: the rows may load before the dependency wait
+  float scale_log2;
+};
+constexpr int kLThreads = 192;   // producer, MMA, four epilogue warps
+constexpr int kLAcc = 4;         // TMEM accumulators of 128 columns
+constexpr int kLStages = 4;
+
+template <int D>
+__global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParams p,
+                                                                  const __grid_constant__ CUtensorMap kmap,
+                                                                  const __grid_constant__ CUtensorMap qmap) {
+  constexpr int STAGES = kLStages;
+  constexpr uint32_t KHALF = kSKeys * 128;   // one 64-column half of a K tile
+  constexpr uint32_t KTILE = kSKeys * D * 2;
+  constexpr uint32_t QHALF = 128 * 128;      // one 64-column half of the 128 window rows
+  constexpr uint32_t QTILE = 128 * D * 2;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t* full_bar = reinterpret_cast<uint64_t*>(smem);
+  uint64_t* empty_bar = full_bar + STAGES;
+  uint64_t* tfull_bar = empty_bar + STAGES;    // [kLAcc]
+  uint64_t* tempty_bar = tfull_bar + kLAcc;    // [kLAcc]
+  uint64_t* qfull_bar = tempty_bar + kLAcc;    // [2]
+  uint64_t* qempty_bar = qfull_bar + 2;        // [2]
+  uint64_t* drain_bar = qempty_bar + 2;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain_bar + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+  int* last_flag = const_cast<int*>(abort_flag) + 1;
+  uint8_t* qbuf = smem + 1024;                 // 2 x QTILE
+  uint8_t* kstage = qbuf + 2 * QTILE;          // STAGES x KTILE
+
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int tpu = p.tiles_per_unit, tpc = p.tiles_per_cta;
+  const int first = blockIdx.x * tpc;
+  const int n = max(0, min(tpc, p.total_tiles - first));
+
+  if (tid == 0) {
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(&full_bar[s], 1);
+      mbar_init(&empty_bar[s], 1);
+    }
+    for (int a = 0; a < kLAcc; ++a) {
+      mbar_init(&tfull_bar[a], 1);
+      mbar_init(&tempty_bar[a], 4);
+    }
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&qfull_bar[i], 1);
+      mbar_init(&qempty_bar[i], 1);
+    }
+    mbar_init(drain_bar, 1);
+    *abort_flag = 0;
+    mbar_fence_init();
+  }
+  if (warp == 1) {
+    tmem_alloc(tmem_slot, kLAcc * 128);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- producer
+    allow_dependent_launch();
+    if (lane == 0) {
+      tma_prefetch_map(&kmap);
+      tma_prefetch_map(&qmap);
+    }
+    int k_issued = 0;
+    auto issue_k = [&](int i) -> bool {
+      bool ok = true;
+      if (lane == 0) {
+        const int g = first + i, unit = g / tpu, tt = g - unit * tpu;
+        const int s = i % STAGES;
+        if (i >= STAGES) ok = mbar_wait(&empty_bar[s], ((i / STAGES) & 1) ^ 1, p.status, abort_flag);
+        if (ok) {
+          uint8_t* st = kstage + s * KTILE;
+          mbar_arrive_expect_tx(&full_bar[s], KTILE);
+#pragma unroll
+          for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * KHALF, &kmap, &full_bar[s], 64 * h, kSKeys * tt, unit);
+          k_issued = i + 1;
+        }
+      }
+      return __shfl_sync(0xffffffffu, ok, 0);
+    };
+    // context K tiles stream before the grid-dependency wait; the window rows after it
+    // (before it as well when the caller says they were written earlier)
+    const int pre = p.window_ready ? 0 : min(n, STAGES);
+    for (int i = 0; i < pre; ++i) issue_k(i);
+    if (!p.window_ready) grid_dependency_wait();
+    int cur_unit = -1, qcount = 0;
+    for (int i = 0; i < n; ++i) {
+      const int unit = (first + i) / tpu;
+      if (unit != cur_unit) {
+        const int qs = qcount & 1;
+        bool ok = true;
+        if (lane == 0) {
+          // rows unit*nq_rows .. +127 (past nq_rows: the next unit's rows or zero fill, whose
+          // results are discarded)
+          if (qcount >= 2) ok = mbar_wait(&qempty_bar[qs], ((qcount >> 1) - 1) & 1, p.status, abort_flag);
+          if (ok) {
+            uint8_t* qb = qbuf + qs * QTILE;
+            mbar_arrive_expect_tx(&qfull_bar[qs], QTILE);
+#pragma unroll
+            for (int h = 0; h < D / 64; ++h) tma_load_2d(qb + h * QHALF, &qmap, &qfull_bar[qs], 64 * h, unit * p.nq_rows);
+          }
+        }
+        if (!__shfl_sync(0xffffffffu, ok, 0)) break;
+        cur_unit = unit;
+        ++qcount;
+      }
+      if (i >= pre && !issue_k(i)) break;
+    }
+    if (lane == 0 && *abort_flag) {   // no copy may land in shared memory after the CTA exits
+      for (int t = max(0, k_issued - STAGES); t < k_issued; ++t)
+        mbar_wait(&full_bar[t % STAGES], (t / STAGES) & 1, p.status, nullptr);
+      for (int q = max(0, qcount - 2); q < qcount; ++q) mbar_wait(&qfull_bar[q & 1], (q >> 1) & 1, p.status, nullptr);
+    }
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    allow_dependent_launch();
+    if (lane == 0) {
+      constexpr uint32_t idesc = umma_idesc_bf16(128, kSKeys);
+      int cur_unit = -1, qcount = 0;
+      for (int i = 0; i < n; ++i) {
+        const int g = first + i, unit = g / tpu;
+        const bool unit_ends = (i == n - 1) || ((g + 1) % tpu == 0);
+        if (unit != cur_unit) {
+          if (!mbar_wait(&qfull_bar[qcount & 1], (qcount >> 1) & 1, p.status, abort_flag)) break;
+          cur_unit = unit;
+          ++qcount;
+        }
+        const int qs = (qcount - 1) & 1;
+        const int s = i % STAGES;
+        if (!mbar_wait(&full_bar[s], (i / STAGES) & 1, p.status, abort_flag)) break;
+        const int acc = i % kLAcc;
+        if (i >= kLAcc && !mbar_wait(&tempty_bar[acc], ((i / kLAcc) & 1) ^ 1, p.status, abort_flag)) break;
+        tc_fence_after();
+        const uint32_t a_base = smem_u32(qbuf + qs * QTILE);
+        const uint32_t b_base = smem_u32(kstage + s * KTILE);
+        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * 128);
+#pragma unroll
+        for (int ks = 0; ks < D / 16; ++ks) {
+          const uint32_t koff = (ks & 3) * 32;
+          const uint64_t adesc = umma_desc_sw128(a_base + (ks >> 2) * QHALF + koff);
+          const uint64_t bdesc = umma_desc_sw128(b_base + (ks >> 2) * KHALF + koff);
+          tc_mma_bf16(d_tmem, adesc, bdesc, idesc, ks > 0 ? 1u : 0u);
+        }
+        tc_commit(&empty_bar[s]);
+        tc_commit(&tfull_bar[acc]);
+        if (unit_ends) tc_commit(&qempty_bar[qs]);
+      }
+      tc_commit(drain_bar);
+      mbar_wait(drain_bar, 0, p.status, nullptr);
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue: one row per thread
+    grid_dependency_wait();
+    allow_dependent_launch();
+    const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
+    const int row = quad * 32 + lane;
+    const int pw = p.t_ctx - p.window + row % p.window;   // last key the row sees
+    const int first_masked = p.t_ctx - p.window;          // keys past it are hidden from some row
+    float m = -INFINITY, l = 0.f;                          // log2 units
+    // after a wait gives up, a warp keeps walking its tiles without touching TMEM, so that
+    // all four warps still meet at every unit-end barrier
+    bool alive = true;
+    for (int i = 0; i < n; ++i) {
+      const int g = first + i, unit = g / tpu, tt = g - unit * tpu;
+      const int acc = i % kLAcc;
+      alive = __all_sync(0xffffffffu, alive && mbar_wait(&tfull_bar[acc], (i / kLAcc) & 1, p.status, abort_flag));
+      if (alive) {
+        tc_fence_after();
+        const int key0 = kSKeys * tt;
+        const bool masked = key0 + kSKeys - 1 > first_masked;
+        const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * 128);
+#pragma unroll
+        for (int c0 = 0; c0 < kSKeys; c0 += 64) {
+          float v[64];
+          tc_ld_32cols(taddr + c0, *reinterpret_cast<float(*)[32]>(&v[0]));
+          tc_ld_32cols(taddr + c0 + 32, *reinterpret_cast<float(*)[32]>(&v[32]));
+          tc_wait_ld();
+          if (masked) {
+#pragma unroll
+            for (int j = 0; j < 64; ++j) v[j] = key0 + c0 + j <= pw ? v[j] : -INFINITY;
+          }
+          float mx0 = fmaxf(v[0], v[1]), mx1 = fmaxf(v[2], v[3]);
+#pragma unroll
+          for (int j = 4; j < 64; j += 4) {
+            mx0 = fmaxf(mx0, fmaxf(v[j], v[j + 1]));
+            mx1 = fmaxf(mx1, fmaxf(v[j + 2], v[j + 3]));
+          }
+          const float mxs = fmaxf(mx0, mx1) * p.scale_log2;
+          if (mxs > m) {
+            l *= fast_exp2(m - mxs);                 // m = -inf: l is still 0
+            m = mxs;
+          }
+          const float2 cc = make_float2(p.scale_log2, p.scale_log2);
+          const float2 nm = make_float2(m == -INFINITY ? 0.f : -m, m == -INFINITY ? 0.f : -m);
+          float2 a0 = make_float2(0.f, 0.f), a1 = a0;
+#pragma unroll
+          for (int j = 0; j < 64; j += 4) {
+            const float2 x0 = ffma2(make_float2(v[j], v[j + 1]), cc, nm);
+            const float2 x1 = ffma2(make_float2(v[j + 2], v[j + 3]), cc, nm);
+            a0 = fadd2(a0, make_float2(fast_exp2(x0.x), fast_exp2(x0.y)));
+            a1 = fadd2(a1, make_float2(fast_exp2(x1.x), fast_exp2(x1.y)));
+          }
+          l += (a0.x + a0.y) + (a1.x + a1.y);
+        }
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&tempty_bar[acc]);
+      }
+      if (i != n - 1 && (g + 1) % tpu != 0) continue;
+      // ------------------------------------------------------------ end of this CTA's part of the unit
+      const int c_first = (unit * tpu) / tpc, c_last = (unit * tpu + tpu - 1) / tpc;
+      const int n_seg = c_last - c_first + 1;
+      const size_t row0 = (size_t)unit * p.nq_rows;
+      if (n_seg == 1) {
+        if (alive && row < p.nq_rows) p.lse[row0 + row] = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
+      } else {
+        float2* seg = p.part + (size_t)unit * p.max_seg * 128;
+        if (alive) seg[(size_t)((int)blockIdx.x - c_first) * 128 + row] = make_float2(m, l);
+        __threadfence();
+        named_bar(1, 128);
+        if (row == 0) *last_flag = alive && atomicAdd(&p.counters[unit], 1) == n_seg - 1;
+        named_bar(1, 128);
+        if (*last_flag) {
+          __threadfence();
+          float M = -INFINITY;
+          for (int k = 0; k < n_seg; ++k) M = fmaxf(M, __ldcg(&seg[(size_t)k * 128 + row].x));
+          float L = 0.f;
+          for (int k = 0; k < n_seg; ++k) {
+            const float2 ml = __ldcg(&seg[(size_t)k * 128 + row]);
+            L += ml.x == -INFINITY ? 0.f : ml.y * fast_exp2(ml.x - M);
+          }
+          if (row < p.nq_rows) p.lse[row0 + row] = L > 0.f ? (M + log2f(L)) * kLn2 : -INFINITY;
+          if (row == 0) p.counters[unit] = 0;
+        }
+        named_bar(1, 128);                        // last_flag is free for the next unit
+      }
+      m = -INFINITY;
+      l = 0.f;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc(tmem_base, kLAcc * 128);
 }
 
 // ============================================================================ top-B select
@@ -1284,22 +1578,47 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   }
   plan->score_bytes = plan->need_scores ? align_up((size_t)units * plan->n_mid_pad * 4, 256) : 0;
   plan->lse_bytes = align_up((size_t)s.batch * s.h_q * window * 4, 256);
-  bd_shape ls = s;
-  ls.t_ctx = s.t_ctx - window;
-  // self mode runs the window LSE through the lse-only verify kernel (at most 128 query
-  // rows per KV head); carry mode does not need it
-  plan->self_mode = verify_plan(ls, window, false, &plan->lse_plan);
+  // self mode's window LSE (carry mode does not need it): window_lse_kernel on the tensor
+  // cores for uniform lengths and up to 128 window rows per KV head, else the lse-only
+  // verify kernel (per-sequence lengths)
+  plan->lse_tc = s.seq_lens == nullptr && plan->nq_rows <= 128 && (long)units * plan->nq_rows >= 128;
+  if (plan->lse_tc) {
+    const int tpu = (s.t_ctx + kSKeys - 1) / kSKeys;
+    const long total = (long)units * tpu;
+    if (total >= (1L << 31)) return false;
+    int grid = (int)std::max<long>(1, std::min<long>(total, current_sm_count()));
+    const int tpc = (int)((total + grid - 1) / grid);
+    grid = (int)((total + tpc - 1) / tpc);
+    int max_seg = 1;
+    for (long u = 0; u < units; ++u)
+      max_seg = std::max(max_seg, (int)((u * tpu + tpu - 1) / tpc - (u * tpu) / tpc + 1));
+    plan->lse_tiles_per_unit = tpu;
+    plan->lse_total_tiles = (int)total;
+    plan->lse_tiles_per_cta = tpc;
+    plan->lse_grid = grid;
+    plan->lse_max_seg = max_seg;
+    plan->lse_smem_bytes = 2048 + (size_t)2 * 128 * s.head_dim * 2 + (size_t)kLStages * kSKeys * s.head_dim * 2;
+    plan->lse_part_bytes = max_seg > 1 ? align_up((size_t)units * max_seg * 128 * sizeof(float2), 256) : 0;
+    plan->self_mode = true;
+  } else {
+    bd_shape ls = s;
+    ls.t_ctx = s.t_ctx - window;
+    plan->self_mode = verify_plan(ls, window, false, &plan->lse_plan);
+  }
   return true;
 }
 
 size_t select_region_bytes(const bd_shape& s, const SelectPlan& plan) {
+  if (!plan.self_mode) return plan.score_bytes;
   bd_shape ls = s;
-  return plan.score_bytes + (plan.self_mode ? plan.lse_bytes + verify_partials_bytes(ls, plan.lse_plan) : 0);
+  ls.t_ctx = s.t_ctx - plan.nq_rows / std::max(1, s.h_q / s.h_kv);
+  return plan.score_bytes + plan.lse_bytes +
+         (plan.lse_tc ? plan.lse_part_bytes : verify_partials_bytes(ls, plan.lse_plan));
 }
 
 cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void* k_cache,
                           const void* q_window, const float* window_lse, int window, int budget,
-                          int n_sink, int n_recent, int chunk, int32_t* idx_out, int32_t* count_out,
+                          int n_sink, int n_recent, int chunk, unsigned flags, int32_t* idx_out, int32_t* count_out,
                           void* ws_region, int* counters, int* status, cudaStream_t stream) {
   const int units = s.batch * s.h_kv;
   uint8_t* region = static_cast<uint8_t*>(ws_region);
@@ -1307,12 +1626,40 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
   cudaError_t err;
   if (plan.need_scores) {
     const float* lse = window_lse;
-    if (lse == nullptr) {   // self mode: window LSE over [0, p_w] through the verify kernel
+    if (lse == nullptr) {   // self mode: window LSE over [0, p_w]
       float* lse_buf = reinterpret_cast<float*>(region + plan.score_bytes);
-      bd_shape ls = s;
-      ls.t_ctx = s.t_ctx - window;
-      err = launch_verify(ls, plan.lse_plan, window, q_window, k_cache, nullptr, nullptr, lse_buf,
-                          region + plan.score_bytes + plan.lse_bytes, counters, status, stream, -window);
+      if (plan.lse_tc) {
+        CUtensorMap lkmap, lqmap;
+        err = make_cache_map(&lkmap, k_cache, units, s.t_cap, s.t_ctx, s.head_dim, kSKeys);
+        if (err != cudaSuccess) return err;
+        err = make_rows_map(&lqmap, q_window, (long long)units * plan.nq_rows, s.head_dim, 128);
+        if (err != cudaSuccess) return err;
+        LseParams lp;
+        lp.lse = lse_buf;
+        lp.part = reinterpret_cast<float2*>(region + plan.score_bytes + plan.lse_bytes);
+        lp.counters = counters;
+        lp.status = status;
+        lp.nq_rows = plan.nq_rows;
+        lp.window = window;
+        lp.t_ctx = s.t_ctx;
+        lp.tiles_per_unit = plan.lse_tiles_per_unit;
+        lp.total_tiles = plan.lse_total_tiles;
+        lp.tiles_per_cta = plan.lse_tiles_per_cta;
+        lp.max_seg = plan.lse_max_seg;
+        lp.window_ready = (flags & BD_SELECT_WINDOW_READY) ? 1 : 0;
+        lp.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
+        void* lfn = s.head_dim == 64 ? reinterpret_cast<void*>(&window_lse_kernel<64>)
+                                     : reinterpret_cast<void*>(&window_lse_kernel<128>);
+        err = cudaFuncSetAttribute(lfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.lse_smem_bytes);
+        if (err != cudaSuccess) return err;
+        void* largs[] = {&lp, &lkmap, &lqmap};
+        err = launch_kernel(lfn, dim3(plan.lse_grid), dim3(kLThreads), plan.lse_smem_bytes, stream, largs, 0);
+      } else {
+        bd_shape ls = s;
+        ls.t_ctx = s.t_ctx - window;
+        err = launch_verify(ls, plan.lse_plan, window, q_window, k_cache, nullptr, nullptr, lse_buf,
+                            region + plan.score_bytes + plan.lse_bytes, counters, status, stream, -window);
+      }
       if (err != cudaSuccess) return err;
       lse = lse_buf;
     }
@@ -1342,6 +1689,7 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
     p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
     p.seq_lens = s.seq_lens;
     p.h_kv = s.h_kv;
+    p.window_ready = (flags & BD_SELECT_WINDOW_READY) ? 1 : 0;
     void* fn = score_fn(s.head_dim, plan.nq_pad, s.seq_lens != nullptr).fn;
     err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
     if (err != cudaSuccess) return err;

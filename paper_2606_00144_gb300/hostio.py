@@ -154,7 +154,8 @@ class HostStepIO:
             for l in L:
                 st, k_cache, _, carry = self.layers[l]
                 self._bind(l, vout)
-                st.select(k_cache, vin[f"q_win{l}"], vin[f"lse{l}"] if carry else None)
+                # the slot's queries landed before the previous step's first draft pass
+                st.select(k_cache, vin[f"q_win{l}"], vin[f"lse{l}"] if carry else None, window_ready=True)
             cs.wait_event(rows_ready)
             if s + 1 < n_steps:
                 cs.wait_event(q_next)

@@ -45,9 +45,12 @@ class SpecStep:
         return cls(wl.batch, wl.h_q, wl.h_kv, wl.head_dim, wl.t_ctx, wl.t_cap, b, wl.n_sink, r,
                    wl.window, wl.gamma, chunk, device)
 
-    def select(self, k_cache, q_win, window_lse=None, stream=None):
+    def select(self, k_cache, q_win, window_lse=None, stream=None, window_ready=False):
+        """window_ready: q_win and window_lse were not written by the kernel launched just
+        before this call (BD_SELECT_WINDOW_READY), so the queries may load while it finishes."""
         B.bd_select_budget(self.shape, k_cache, q_win, window_lse, self.window, self.budget, self.n_sink,
-                           self.n_recent, self.chunk, self.idx, self.count, self.ws, stream)
+                           self.n_recent, self.chunk, self.idx, self.count, self.ws, stream,
+                           flags=B.BD_SELECT_WINDOW_READY if window_ready else 0)
 
     def draft(self, j, q_j, k_cache, v_cache, stream=None, view_ready=False):
         """Draft pass j.  view_ready: the selection was not written by the kernel launched

@@ -62,9 +62,9 @@ def draft(lib, s, q=A, k=A, v=A, idx=A, cnt=A, budget=32, j=0, o=A, lse=A, ws=A,
 
 
 def select(lib, s, k=A, qw=A, lse=A, window=32, budget=40, sink=4, recent=8, chunk=1, idx=A, cnt=A, ws=A,
-           nbytes=1 << 20):
-    return lib.bd_select_budget(ctypes.byref(s), k, qw, lse, window, budget, sink, recent, chunk, idx, cnt, ws,
-                                nbytes, None)
+           nbytes=1 << 20, flags=0):
+    return lib.bd_select_budget(ctypes.byref(s), k, qw, lse, window, budget, sink, recent, chunk, flags, idx, cnt,
+                                ws, nbytes, None)
 
 
 def test_verify_validation(lib):
@@ -97,6 +97,7 @@ def test_select_validation(lib):
     assert select(lib, shape(), window=101) == INVALID                # window > t_ctx
     assert select(lib, shape(), budget=10, sink=4, recent=8) == INVALID   # sink + recent > budget
     assert select(lib, shape(), chunk=0) == INVALID
+    assert select(lib, shape(), flags=2) == INVALID                   # unknown flag bits
     assert select(lib, shape(), sink=-1) == INVALID
     assert select(lib, shape(), lse=A + 1) == MISALIGNED
     assert select(lib, shape(h_q=16, h_kv=1), window=32) == UNSUPPORTED  # 512 window rows > 256

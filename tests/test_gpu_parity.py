@@ -52,7 +52,9 @@ def run_and_check(wl, inp, h, budgets=None, modes=("carry", "self"), chunk=1, ch
                 idx_ref[b, kv, : keep.size] = keep
                 cnt_ref[b, kv] = keep.size
         for mode in modes:
-            st.select(inp.k_cache, inp.q_win, lse_dev if mode == "carry" else None)
+            # both orders of the window-query load: early (BD_SELECT_WINDOW_READY) in carry
+            # mode, after the dependency wait in self mode
+            st.select(inp.k_cache, inp.q_win, lse_dev if mode == "carry" else None, window_ready=mode == "carry")
             torch.cuda.synchronize()
             nd = check_selection(st.idx, st.count, idx_ref, cnt_ref, score_ref, t, budget, wl.n_sink, n_recent,
                                  chunk, what=f"{tag} B={budget} {mode}")
