@@ -275,12 +275,17 @@ bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
   const int g = s.h_q / s.h_kv;
   if (g < 1 || g > 8 || !pick(s.head_dim, draft_group_instance(g))) return false;
   const long entries = (long)budget + n_steps;
-  // one tile per CTA up to a cluster of 8, but no more CTAs than one wave holds (about three
-  // single-stage CTAs per SM): a second wave would repeat the whole latency chain of a pass
+  // one tile per CTA up to a cluster of 8, but no more CTAs than one wave holds at the
+  // occupancy the slice's stage count gives (three single-stage or two double-buffered
+  // CTAs per SM, see launch_draft): a second wave would repeat the pass's whole latency chain
   const long units = (long)s.batch * s.h_kv;
-  const long wave = 3L * current_sm_count();
+  const long sms = current_sm_count();
   int n_split = (int)std::min<long>((entries + kDRows - 1) / kDRows, kDMaxCluster);
-  n_split = (int)std::min<long>(n_split, std::max<long>(1, wave / std::max<long>(1, units)));
+  for (; n_split > 1; --n_split) {
+    const long rps = (entries + n_split - 1) / n_split, ctas = units * n_split;
+    const bool dbuf = (rps > kDRows && ctas <= 2 * sms) || rps > 2 * kDRows;
+    if (ctas <= (dbuf ? 2 : 3) * sms) break;
+  }
   n_split = std::max(n_split, 1);
   plan->n_entries_max = (int)entries;
   plan->rows_per_split = (int)((entries + n_split - 1) / n_split);
