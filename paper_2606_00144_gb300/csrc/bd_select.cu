@@ -368,13 +368,13 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
 // Self mode's normalisers: lse_r = log sum_{k <= p_w} exp(q_r . k_k / sqrt(d)) for the G*W
 // window rows r = h*W + w of every unit (p_w = t_ctx - W + w).  The contraction of
 // score_kernel with its operands swapped: the unit's window rows are the A operand (M =
-// 128 rows = the TMEM lanes) and a 128-key K tile the B operand (N = 128 columns), so each
-// of the four epilogue warps' threads owns one window row and keeps that row's online
-// log-sum-exp in registers, with no cross-thread reduction.  Persistent CTAs (one per SM)
+// 128 rows = the TMEM lanes) and a 128-key K tile the B operand (N = 128 columns), so a
+// row's online log-sum-exp stays inside the two threads that own it (one per 64-column
+// half of the TMEM row), with no reduction across lanes.  Persistent CTAs (one per SM)
 // take contiguous ranges of the (unit, 128-key tile) list: warp 0 streams K tiles (TMA,
 // 4-stage ring) and the unit's rows (two buffers), warp 1 issues the MMAs into four TMEM
-// accumulators, warps 2-5 reduce.  A unit split over several CTAs merges the segments'
-// (max, sum) pairs in the CTA that finishes it last.
+// accumulators, warps 2-9 reduce (two warps per TMEM lane quarter).  A unit split over
+// several CTAs merges the segments' (max, sum) pairs in the CTA that finishes it last.
 struct LseParams {
   float* lse;          // [units * nq_rows] natural log
   float2* part;        // [units][max_seg][128]: a segment's (running max in log2 units, sum)
@@ -384,7 +384,7 @@ struct LseParams {
   int window_ready;    // BD_SELECT_WINDOW_READY: the rows may load before the dependency wait
   float scale_log2;
 };
-constexpr int kLThreads = 192;   // producer, MMA, four epilogue warps
+constexpr int kLThreads = 320;   // producer, MMA, eight epilogue warps (two per TMEM lane quarter)
 constexpr int kLAcc = 4;         // TMEM accumulators of 128 columns
 constexpr int kLStages = 4;
 
@@ -411,6 +411,7 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
   int* last_flag = const_cast<int*>(abort_flag) + 1;
   uint8_t* qbuf = smem + 1024;                 // 2 x QTILE
   uint8_t* kstage = qbuf + 2 * QTILE;          // STAGES x KTILE
+  float2* ml_s = reinterpret_cast<float2*>(kstage + STAGES * KTILE);   // [2][128] the column halves' (m, l)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int tpu = p.tiles_per_unit, tpc = p.tiles_per_cta;
@@ -424,7 +425,7 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
     }
     for (int a = 0; a < kLAcc; ++a) {
       mbar_init(&tfull_bar[a], 1);
-      mbar_init(&tempty_bar[a], 4);
+      mbar_init(&tempty_bar[a], 8);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(&qfull_bar[i], 1);
@@ -538,16 +539,17 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
       mbar_wait(drain_bar, 0, p.status, nullptr);
     }
   } else {
-    // ---------------------------------------------------------------- epilogue: one row per thread
+    // ---------------------------------------------------------------- epilogue: a row's half per thread
     grid_dependency_wait();
     allow_dependent_launch();
     const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
+    const int half = (warp - 2) >> 2;           // warps 2-5: columns 0-63, warps 6-9: 64-127
     const int row = quad * 32 + lane;
     const int pw = p.t_ctx - p.window + row % p.window;   // last key the row sees
     const int first_masked = p.t_ctx - p.window;          // keys past it are hidden from some row
     float m = -INFINITY, l = 0.f;                          // log2 units
     // after a wait gives up, a warp keeps walking its tiles without touching TMEM, so that
-    // all four warps still meet at every unit-end barrier
+    // all eight warps still meet at every unit-end barrier
     bool alive = true;
     for (int i = 0; i < n; ++i) {
       const int g = first + i, unit = g / tpu, tt = g - unit * tpu;
@@ -558,8 +560,8 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
         const int key0 = kSKeys * tt;
         const bool masked = key0 + kSKeys - 1 > first_masked;
         const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + (uint32_t)(acc * 128);
-#pragma unroll
-        for (int c0 = 0; c0 < kSKeys; c0 += 64) {
+        {
+          const int c0 = 64 * half;
           float v[64];
           tc_ld_32cols(taddr + c0, *reinterpret_cast<float(*)[32]>(&v[0]));
           tc_ld_32cols(taddr + c0 + 32, *reinterpret_cast<float(*)[32]>(&v[32]));
@@ -597,19 +599,30 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
       }
       if (i != n - 1 && (g + 1) % tpu != 0) continue;
       // ------------------------------------------------------------ end of this CTA's part of the unit
+      // the two column halves of each row meet first
+      ml_s[half * 128 + row] = alive ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
+      named_bar(1, 256);
       const int c_first = (unit * tpu) / tpc, c_last = (unit * tpu + tpu - 1) / tpc;
       const int n_seg = c_last - c_first + 1;
       const size_t row0 = (size_t)unit * p.nq_rows;
-      if (n_seg == 1) {
-        if (alive && row < p.nq_rows) p.lse[row0 + row] = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
-      } else {
-        float2* seg = p.part + (size_t)unit * p.max_seg * 128;
-        if (alive) seg[(size_t)((int)blockIdx.x - c_first) * 128 + row] = make_float2(m, l);
+      float2* seg = p.part + (size_t)unit * p.max_seg * 128;
+      if (half == 0) {
+        const float2 o = ml_s[128 + row];
+        const float M2 = fmaxf(m, o.x);
+        l = (m == -INFINITY ? 0.f : l * fast_exp2(m - M2)) + (o.x == -INFINITY ? 0.f : o.y * fast_exp2(o.x - M2));
+        m = M2;
+        if (n_seg == 1) {
+          if (alive && row < p.nq_rows) p.lse[row0 + row] = l > 0.f ? (m + log2f(l)) * kLn2 : -INFINITY;
+        } else if (alive) {
+          seg[(size_t)((int)blockIdx.x - c_first) * 128 + row] = make_float2(m, l);
+        }
+      }
+      if (n_seg > 1) {
         __threadfence();
-        named_bar(1, 128);
-        if (row == 0) *last_flag = alive && atomicAdd(&p.counters[unit], 1) == n_seg - 1;
-        named_bar(1, 128);
-        if (*last_flag) {
+        named_bar(1, 256);
+        if (half == 0 && row == 0) *last_flag = alive && atomicAdd(&p.counters[unit], 1) == n_seg - 1;
+        named_bar(1, 256);
+        if (half == 0 && *last_flag) {
           __threadfence();
           float M = -INFINITY;
           for (int k = 0; k < n_seg; ++k) M = fmaxf(M, __ldcg(&seg[(size_t)k * 128 + row].x));
@@ -621,8 +634,8 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
           if (row < p.nq_rows) p.lse[row0 + row] = L > 0.f ? (M + log2f(L)) * kLn2 : -INFINITY;
           if (row == 0) p.counters[unit] = 0;
         }
-        named_bar(1, 128);                        // last_flag is free for the next unit
       }
+      named_bar(1, 256);                          // ml_s and last_flag are free for the next unit
       m = -INFINITY;
       l = 0.f;
     }
@@ -1597,7 +1610,8 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
     plan->lse_tiles_per_cta = tpc;
     plan->lse_grid = grid;
     plan->lse_max_seg = max_seg;
-    plan->lse_smem_bytes = 2048 + (size_t)2 * 128 * s.head_dim * 2 + (size_t)kLStages * kSKeys * s.head_dim * 2;
+    plan->lse_smem_bytes = 2048 + (size_t)2 * 128 * s.head_dim * 2 + (size_t)kLStages * kSKeys * s.head_dim * 2 +
+                           2 * 128 * sizeof(float2);
     plan->lse_part_bytes = max_seg > 1 ? align_up((size_t)units * max_seg * 128 * sizeof(float2), 256) : 0;
     plan->self_mode = true;
   } else {
