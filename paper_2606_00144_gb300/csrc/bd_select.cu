@@ -1,4 +1,6 @@
-// KV-budget selection (Sec. 3.4 TopKChunks; Algorithm 2, sparsify) in two kernels:
+// KV-budget selection (Sec. 3.4 TopKChunks; Algorithm 2, sparsify) in two kernels (three
+// in self mode, where window_lse_kernel first computes the window rows' normalisers, see
+// its own comment below):
 //
 // score_kernel  (tcgen05)  score[k] = sum_{h in group, w < W, k <= p_w} exp2(s_{h,w,k} log2e/sqrt(d)
 //               - lse_{h,w} log2e) for every middle key k.  Keys sit on the M side of the
