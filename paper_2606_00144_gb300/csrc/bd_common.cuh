@@ -147,6 +147,15 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* s
 // ---------------------------------------------------------------------------------------
 // TMA (tiled tensor copies global -> shared, completion counted on an mbarrier)
 // ---------------------------------------------------------------------------------------
+// Starts [p, p + bytes) on its way into L2 (no L1 allocation, nothing to wait for): safe
+// before a grid-dependency wait on data the preceding kernel may still write, since L2 is
+// where those writes land and the real load after the wait reads through it.  One line per
+// thread of [0, n_threads).
+__device__ __forceinline__ void prefetch_lines_l2(const void* p, size_t bytes, int tid, int n_threads) {
+  const char* c = static_cast<const char*>(p);
+  for (size_t off = (size_t)tid * 128; off < bytes; off += (size_t)n_threads * 128)
+    asm volatile("prefetch.global.L2 [%0];" ::"l"(reinterpret_cast<uint64_t>(c + off)) : "memory");
+}
 __device__ __forceinline__ void tma_prefetch_map(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }

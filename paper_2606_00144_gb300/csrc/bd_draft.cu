@@ -76,6 +76,8 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   constexpr uint32_t HALF_BYTES = kDRows * 128;
   constexpr int CH = D / 8;                    // 16-byte chunks per row
   const bool early = (p.flags & BD_DRAFT_VIEW_READY) != 0;
+  // the pass's queries (read after the wait below) on their way into L2 meanwhile
+  prefetch_lines_l2(p.q + (size_t)blockIdx.y * p.g * D, (size_t)p.g * D * 2, threadIdx.x, kDThreads);
   if (!early) {
     grid_dependency_wait();
     allow_dependent_launch();

@@ -200,7 +200,14 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     // they were written earlier (then queries and tiles interleave from the start)
     const int pre = p.window_ready ? 0 : min(n, STAGES);
     for (int i = 0; i < pre; ++i) issue_k(i);
-    if (!p.window_ready) grid_dependency_wait();
+    if (!p.window_ready) {
+      if (n > 0) {   // the first unit's queries on their way into L2 meanwhile
+        int u0, t0;
+        locate(first, u0, t0);
+        prefetch_lines_l2(p.q_win + (size_t)u0 * p.nq_rows * D, (size_t)p.nq_rows * D * 2, lane, 32);
+      }
+      grid_dependency_wait();
+    }
     int cur_unit = -1, qcount = 0;
     for (int i = 0; i < n; ++i) {
       const int g = first + i;
@@ -276,6 +283,8 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
     }
   } else {
     // ---------------------------------------------------------------- epilogue (2 groups of 4 warps)
+    if (!RAGGED && n > 0 && warp == 2)           // the first unit's window LSE into L2 meanwhile
+      prefetch_lines_l2(p.lse_win + (size_t)(first / p.tiles_per_unit) * p.nq_rows, (size_t)p.nq_rows * 4, lane, 32);
     grid_dependency_wait();                      // the window LSE is carried from earlier kernels
     allow_dependent_launch();
     const int grp = (warp - 2) >> 2;            // group g: warps 2+4g .. 5+4g; tiles i % 4 == g
@@ -378,6 +387,7 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
 // accumulators, warps 2-9 reduce (two warps per TMEM lane quarter).  A unit split over
 // several CTAs merges the segments' (max, sum) pairs in the CTA that finishes it last.
 struct LseParams {
+  const __nv_bfloat16* q_win;   // [units * nq_rows][D] (read by TMA; prefetched through this pointer)
   float* lse;          // [units * nq_rows] natural log
   float2* part;        // [units][max_seg][128]: a segment's (running max in log2 units, sum)
   int* counters;       // [units] arrival counters (left zero)
@@ -474,7 +484,11 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
     // (before it as well when the caller says they were written earlier)
     const int pre = p.window_ready ? 0 : min(n, STAGES);
     for (int i = 0; i < pre; ++i) issue_k(i);
-    if (!p.window_ready) grid_dependency_wait();
+    if (!p.window_ready) {
+      if (n > 0)   // the first unit's rows on their way into L2 meanwhile
+        prefetch_lines_l2(p.q_win + (size_t)(first / tpu) * p.nq_rows * D, (size_t)p.nq_rows * D * 2, lane, 32);
+      grid_dependency_wait();
+    }
     int cur_unit = -1, qcount = 0;
     for (int i = 0; i < n; ++i) {
       const int unit = (first + i) / tpu;
@@ -1651,6 +1665,7 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
         err = make_rows_map(&lqmap, q_window, (long long)units * plan.nq_rows, s.head_dim, 128);
         if (err != cudaSuccess) return err;
         LseParams lp;
+        lp.q_win = static_cast<const __nv_bfloat16*>(q_window);
         lp.lse = lse_buf;
         lp.part = reinterpret_cast<float2*>(region + plan.score_bytes + plan.lse_bytes);
         lp.counters = counters;

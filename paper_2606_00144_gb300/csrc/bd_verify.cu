@@ -213,6 +213,8 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   }
 
   // -------------------------------------------------------------------- consumers
+  if (!p.seq_lens)   // the first unit's queries on their way into L2 while the predecessor finishes
+    prefetch_lines_l2(p.q + (size_t)u_first * p.nq_rows * D, (size_t)p.nq_rows * D * 2, tid, kVConsumers * 32);
   grid_dependency_wait();                        // the queries come from the preceding kernels
   allow_dependent_launch();
   const int wq = warp % WQ, wk = warp / WQ;
