@@ -289,7 +289,6 @@ bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
     if (ctas <= (dbuf ? 2 : 3) * sms) break;
   }
   n_split = std::max(n_split, 1);
-  plan->n_entries_max = (int)entries;
   plan->rows_per_split = (int)((entries + n_split - 1) / n_split);
   plan->n_split = n_split;
   return true;

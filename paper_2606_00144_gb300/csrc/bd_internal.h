@@ -50,7 +50,6 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
 
 // ---------------------------------------------------------------------------- draft
 struct DraftPlan {
-  int n_entries_max;    // budget + step_j + 1
   int n_split;
   int rows_per_split;
 };
