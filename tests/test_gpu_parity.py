@@ -359,6 +359,17 @@ def test_boundary_among_underflowed_scores():
     run_and_check(wl, inp, host(inp), check_steps=False, tag="boundary among zero scores")
 
 
+@pytest.mark.parametrize("d", [64, 128])
+def test_self_mode_whole_units_per_cta(d):
+    """128 (sequence, KV head) units of one 128-key tile each: every CTA of the window-LSE
+    kernel holds whole units, so each unit's normalisers are written directly (no segment
+    merge), next to the split-unit path the longer workloads take."""
+    wl = W.tiny_workload(batch=16, h_q=32, h_kv=8, head_dim=d, t_ctx=120, budget=64, n_sink=4, n_recent=16,
+                         window=32, gamma=2)
+    inp = W.make_layer(wl, 0, "cuda")
+    run_and_check(wl, inp, host(inp), modes=("self",), check_steps=False, tag=f"whole units d{d}")
+
+
 def test_determinism():
     wl = W.WORKLOADS["l8b_4k"]
     inp = W.make_layer(wl, 0, "cuda")
