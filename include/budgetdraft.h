@@ -107,9 +107,10 @@ size_t bd_workspace_size(const bd_shape* shape, int op, int budget, int n_q);
 
 /* bd_select_budget flags. */
 enum {
-  /* q_window (and window_lse) were written before the kernel that immediately precedes
-   * this call on `stream` (not by it: bd_advance, for one, rewrites them in place): the
-   * call may load the window queries while that kernel finishes. */
+  /* q_window, window_lse and the shape's per-sequence lengths (if any) were written
+   * before the kernel that immediately precedes this call on `stream` (not by it:
+   * bd_advance, for one, rewrites all three in place): the call may read them while
+   * that kernel finishes. */
   BD_SELECT_WINDOW_READY = 1
 };
 

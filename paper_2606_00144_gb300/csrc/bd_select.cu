@@ -89,7 +89,9 @@ __global__ void __launch_bounds__(kSThreads, 1) score_kernel(const ScoreParams p
   int* spref = reinterpret_cast<int*>(kstage + STAGES * KTILE);   // [units + 1]
   int total = p.total_tiles, tpc = p.tiles_per_cta;
   if (RAGGED) {
-    grid_dependency_wait();
+    // with BD_SELECT_WINDOW_READY the lengths were settled before the kernel just before
+    // this one too, so the layout (and the streaming) need not wait for it
+    if (!p.window_ready) grid_dependency_wait();
     int* wtot = reinterpret_cast<int*>(smem + 1024);
     const int per = (n_units + kSThreads - 1) / kSThreads;
     const int u0 = min(n_units, tid * per), u1 = min(n_units, u0 + per);

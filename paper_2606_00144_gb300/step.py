@@ -46,8 +46,9 @@ class SpecStep:
                    wl.window, wl.gamma, chunk, device)
 
     def select(self, k_cache, q_win, window_lse=None, stream=None, window_ready=False):
-        """window_ready: q_win and window_lse were not written by the kernel launched just
-        before this call (BD_SELECT_WINDOW_READY), so the queries may load while it finishes."""
+        """window_ready: q_win, window_lse and the per-sequence lengths were not written by the
+        kernel launched just before this call (BD_SELECT_WINDOW_READY), so they may be read
+        while it finishes."""
         B.bd_select_budget(self.shape, k_cache, q_win, window_lse, self.window, self.budget, self.n_sink,
                            self.n_recent, self.chunk, self.idx, self.count, self.ws, stream,
                            flags=B.BD_SELECT_WINDOW_READY if window_ready else 0)

@@ -53,15 +53,24 @@ def test_ragged_lengths_match_per_sequence_oracle(mode):
     ws = bd.Workspace.for_step(shape, budget, W, gamma)
     idx = torch.empty(b, hkv, budget, dtype=torch.int32, device="cuda")
     cnt = torch.empty(b, hkv, dtype=torch.int32, device="cuda")
-    bd.bd_select_budget(shape, inp.k_cache, inp.q_win, lse_d, W, budget, sink, recent, 1, idx, cnt, ws)
-    torch.cuda.synchronize()
     idx_ref = np.full((b, hkv, budget), -1)
     cnt_ref = np.zeros((b, hkv), dtype=np.int64)
+    refs = []
     for i, t in enumerate(lens):
         ir, cr, score = oracle_selection(h["QW"][i:i + 1], h["K"][i:i + 1], lse_ref[i], t, budget, sink, recent)
         idx_ref[i], cnt_ref[i] = ir[0], cr[0]
-        check_selection(idx[i:i + 1], cnt[i:i + 1], ir, cr, score, t, budget, sink, recent, 1,
-                        what=f"{mode} seq {i} T={t}")
+        refs.append((ir, cr, score))
+    # carry mode also with BD_SELECT_WINDOW_READY: the tile layout of the lengths is then
+    # built before the dependency wait
+    for flags in ((0, bd.BD_SELECT_WINDOW_READY) if mode == "carry" else (0,)):
+        idx.fill_(-7)
+        bd.bd_select_budget(shape, inp.k_cache, inp.q_win, lse_d, W, budget, sink, recent, 1, idx, cnt, ws,
+                            flags=flags)
+        torch.cuda.synchronize()
+        for i, t in enumerate(lens):
+            ir, cr, score = refs[i]
+            check_selection(idx[i:i + 1], cnt[i:i + 1], ir, cr, score, t, budget, sink, recent, 1,
+                            what=f"{mode} flags {flags} seq {i} T={t}")
     assert cnt_ref[-1].tolist() == [lens[-1]] * hkv             # B >= T_b keeps everything
     # drafts on the oracle's selection, verify
     idx.copy_(torch.from_numpy(idx_ref).int())
