@@ -1530,6 +1530,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
 #pragma unroll
   for (int r = 0; r < ROWS; ++r) {
     const uint32_t mk = masks[r];
+    if (mk == 0u) continue;                        // warp-uniform: most rows hold no kept item
     if ((mk >> lane) & 1u) out[base + __popc(mk & lt)] = lo + w0 + 32 * r + lane;
     base += __popc(mk);
   }
