@@ -397,12 +397,18 @@ struct LseParams {
   int nq_rows, window, t_ctx, tiles_per_unit, total_tiles, tiles_per_cta, max_seg;
   int window_ready;    // BD_SELECT_WINDOW_READY: the rows may load before the dependency wait
   float scale_log2;
+  const int32_t* seq_lens;   // per-sequence context lengths [batch] (RAGGED instance) or null
+  int h_kv, units;
 };
+constexpr int kLMaxSeg = 8;      // segments of one unit with per-sequence lengths (bounds the partials)
 constexpr int kLThreads = 320;   // producer, MMA, eight epilogue warps (two per TMEM lane quarter)
 constexpr int kLAcc = 4;         // TMEM accumulators of 128 columns
 constexpr int kLStages = 4;
 
-template <int D>
+// RAGGED: per-sequence lengths; every CTA lays out the units' tiles itself (a prefix table in
+// shared memory, as score_kernel's ragged instance does) and the range per CTA is at least
+// tiles_per_cta, which keeps a unit within kLMaxSeg segments.
+template <int D, bool RAGGED>
 __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParams p,
                                                                   const __grid_constant__ CUtensorMap kmap,
                                                                   const __grid_constant__ CUtensorMap qmap) {
@@ -426,11 +432,56 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
   uint8_t* qbuf = smem + 1024;                 // 2 x QTILE
   uint8_t* kstage = qbuf + 2 * QTILE;          // STAGES x KTILE
   float2* ml_s = reinterpret_cast<float2*>(kstage + STAGES * KTILE);   // [2][128] the column halves' (m, l)
+  int* spref = reinterpret_cast<int*>(ml_s + 256);                      // [units + 1] (RAGGED)
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int tpu = p.tiles_per_unit, tpc = p.tiles_per_cta;
+  const int tpu = p.tiles_per_unit;
+  int total = p.total_tiles, tpc = p.tiles_per_cta;
+  if (RAGGED) {
+    // the lengths may come from the kernel just before (bd_advance moves them), unless the
+    // caller says otherwise
+    if (!p.window_ready) grid_dependency_wait();
+    int* wtot = reinterpret_cast<int*>(smem + 512);
+    const int per = (p.units + kLThreads - 1) / kLThreads;
+    const int u0 = min(p.units, tid * per), u1 = min(p.units, u0 + per);
+    auto tiles_of = [&](int u) {
+      return (unit_context(p.seq_lens, u, p.h_kv, p.t_ctx, nullptr) + kSKeys - 1) / kSKeys;
+    };
+    int sum = 0;
+    for (int u = u0; u < u1; ++u) sum += tiles_of(u);
+    int incl = sum;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, incl, off);
+      if (lane >= off) incl += y;
+    }
+    if (lane == 31) wtot[warp] = incl;
+    __syncthreads();
+    int run = incl - sum;
+    for (int w = 0; w < warp; ++w) run += wtot[w];
+    for (int u = u0; u < u1; ++u) {
+      spref[u] = run;
+      run += tiles_of(u);
+    }
+    if (tid == kLThreads - 1) spref[p.units] = run;
+    __syncthreads();
+    total = spref[p.units];
+    tpc = max((total + (int)gridDim.x - 1) / (int)gridDim.x, p.tiles_per_cta);
+  }
   const int first = blockIdx.x * tpc;
-  const int n = max(0, min(tpc, p.total_tiles - first));
+  const int n = max(0, min(tpc, total - first));
+  auto unit_of = [&](int g) {
+    if (!RAGGED) return g / tpu;
+    int lo = 0, hi = p.units - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (spref[mid] <= g) lo = mid;
+      else hi = mid - 1;
+    }
+    return lo;
+  };
+  auto unit_begin = [&](int u) { return RAGGED ? spref[u] : u * tpu; };
+  auto unit_end = [&](int u) { return RAGGED ? spref[u + 1] : (u + 1) * tpu; };
 
   if (tid == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -469,7 +520,7 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
     auto issue_k = [&](int i) -> bool {
       bool ok = true;
       if (lane == 0) {
-        const int g = first + i, unit = g / tpu, tt = g - unit * tpu;
+        const int g = first + i, unit = unit_of(g), tt = g - unit_begin(unit);
         const int s = i % STAGES;
         if (i >= STAGES) ok = mbar_wait(&empty_bar[s], ((i / STAGES) & 1) ^ 1, p.status, abort_flag);
         if (ok) {
@@ -488,12 +539,12 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
     for (int i = 0; i < pre; ++i) issue_k(i);
     if (!p.window_ready) {
       if (n > 0)   // the first unit's rows on their way into L2 meanwhile
-        prefetch_lines_l2(p.q_win + (size_t)(first / tpu) * p.nq_rows * D, (size_t)p.nq_rows * D * 2, lane, 32);
+        prefetch_lines_l2(p.q_win + (size_t)unit_of(first) * p.nq_rows * D, (size_t)p.nq_rows * D * 2, lane, 32);
       grid_dependency_wait();
     }
     int cur_unit = -1, qcount = 0;
     for (int i = 0; i < n; ++i) {
-      const int unit = (first + i) / tpu;
+      const int unit = unit_of(first + i);
       if (unit != cur_unit) {
         const int qs = qcount & 1;
         bool ok = true;
@@ -526,8 +577,8 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
       constexpr uint32_t idesc = umma_idesc_bf16(128, kSKeys);
       int cur_unit = -1, qcount = 0;
       for (int i = 0; i < n; ++i) {
-        const int g = first + i, unit = g / tpu;
-        const bool unit_ends = (i == n - 1) || ((g + 1) % tpu == 0);
+        const int g = first + i, unit = unit_of(g);
+        const bool unit_ends = (i == n - 1) || g + 1 == unit_end(unit);
         if (unit != cur_unit) {
           if (!mbar_wait(&qfull_bar[qcount & 1], (qcount >> 1) & 1, p.status, abort_flag)) break;
           cur_unit = unit;
@@ -563,14 +614,22 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
     const int quad = warp & 3;                  // TMEM lanes quad*32 .. quad*32+31
     const int half = (warp - 2) >> 2;           // warps 2-5: columns 0-63, warps 6-9: 64-127
     const int row = quad * 32 + lane;
-    const int pw = p.t_ctx - p.window + row % p.window;   // last key the row sees
-    const int first_masked = p.t_ctx - p.window;          // keys past it are hidden from some row
+    int pw = p.t_ctx - p.window + row % p.window;         // last key the row sees
+    int first_masked = p.t_ctx - p.window;                // keys past it are hidden from some row
+    int cur_unit = -1;
     float m = -INFINITY, l = 0.f;                          // log2 units
     // after a wait gives up, a warp keeps walking its tiles without touching TMEM, so that
     // all eight warps still meet at every unit-end barrier
     bool alive = true;
     for (int i = 0; i < n; ++i) {
-      const int g = first + i, unit = g / tpu, tt = g - unit * tpu;
+      const int g = first + i, unit = unit_of(g), tt = g - unit_begin(unit);
+      if (RAGGED && unit != cur_unit) {
+        const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 64 ? p.status : nullptr);
+        if (t_u < p.window && tid == 64) record_error(p.status, BD_ERR_INVALID_ARG);
+        pw = t_u - p.window + row % p.window;
+        first_masked = t_u - p.window;
+        cur_unit = unit;
+      }
       const int acc = i % kLAcc;
       alive = __all_sync(0xffffffffu, alive && mbar_wait(&tfull_bar[acc], (i / kLAcc) & 1, p.status, abort_flag));
       if (alive) {
@@ -615,12 +674,12 @@ __global__ void __launch_bounds__(kLThreads, 1) window_lse_kernel(const LseParam
         __syncwarp();
         if (lane == 0) mbar_arrive(&tempty_bar[acc]);
       }
-      if (i != n - 1 && (g + 1) % tpu != 0) continue;
+      if (i != n - 1 && g + 1 != unit_end(unit)) continue;
       // ------------------------------------------------------------ end of this CTA's part of the unit
       // the two column halves of each row meet first
       ml_s[half * 128 + row] = alive ? make_float2(m, l) : make_float2(-INFINITY, 0.f);
       named_bar(1, 256);
-      const int c_first = (unit * tpu) / tpc, c_last = (unit * tpu + tpu - 1) / tpc;
+      const int c_first = unit_begin(unit) / tpc, c_last = (unit_end(unit) - 1) / tpc;
       const int n_seg = c_last - c_first + 1;
       const size_t row0 = (size_t)unit * p.nq_rows;
       float2* seg = p.part + (size_t)unit * p.max_seg * 128;
@@ -1611,26 +1670,34 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
   plan->score_bytes = plan->need_scores ? align_up((size_t)units * plan->n_mid_pad * 4, 256) : 0;
   plan->lse_bytes = align_up((size_t)s.batch * s.h_q * window * 4, 256);
   // self mode's window LSE (carry mode does not need it): window_lse_kernel on the tensor
-  // cores for uniform lengths and up to 128 window rows per KV head, else the lse-only
-  // verify kernel (per-sequence lengths)
-  plan->lse_tc = s.seq_lens == nullptr && plan->nq_rows <= 128 && (long)units * plan->nq_rows >= 128;
+  // cores for up to 128 window rows per KV head (with per-sequence lengths a unit spans at
+  // most kLMaxSeg CTA ranges), else the lse-only verify kernel
+  plan->lse_tc = plan->nq_rows <= 128 && (long)units * plan->nq_rows >= 128;
   if (plan->lse_tc) {
     const int tpu = (s.t_ctx + kSKeys - 1) / kSKeys;
     const long total = (long)units * tpu;
     if (total >= (1L << 31)) return false;
     int grid = (int)std::max<long>(1, std::min<long>(total, current_sm_count()));
-    const int tpc = (int)((total + grid - 1) / grid);
-    grid = (int)((total + tpc - 1) / tpc);
+    int tpc = (int)((total + grid - 1) / grid);
     int max_seg = 1;
-    for (long u = 0; u < units; ++u)
-      max_seg = std::max(max_seg, (int)((u * tpu + tpu - 1) / tpc - (u * tpu) / tpc + 1));
+    if (s.seq_lens) {
+      // the lengths are read on the device: every SM gets a CTA, and the range per CTA is
+      // bounded below so that a unit of tpu tiles spans at most kLMaxSeg ranges
+      grid = current_sm_count();
+      tpc = (tpu + kLMaxSeg - 2) / (kLMaxSeg - 1);
+      max_seg = kLMaxSeg;
+    } else {
+      grid = (int)((total + tpc - 1) / tpc);
+      for (long u = 0; u < units; ++u)
+        max_seg = std::max(max_seg, (int)((u * tpu + tpu - 1) / tpc - (u * tpu) / tpc + 1));
+    }
     plan->lse_tiles_per_unit = tpu;
     plan->lse_total_tiles = (int)total;
     plan->lse_tiles_per_cta = tpc;
     plan->lse_grid = grid;
     plan->lse_max_seg = max_seg;
     plan->lse_smem_bytes = 2048 + (size_t)2 * 128 * s.head_dim * 2 + (size_t)kLStages * kSKeys * s.head_dim * 2 +
-                           2 * 128 * sizeof(float2);
+                           2 * 128 * sizeof(float2) + (s.seq_lens ? align_up((size_t)(units + 1) * 4, 16) : 0);
     plan->lse_part_bytes = max_seg > 1 ? align_up((size_t)units * max_seg * 128 * sizeof(float2), 256) : 0;
     plan->self_mode = true;
   } else {
@@ -1681,9 +1748,14 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
         lp.tiles_per_cta = plan.lse_tiles_per_cta;
         lp.max_seg = plan.lse_max_seg;
         lp.window_ready = (flags & BD_SELECT_WINDOW_READY) ? 1 : 0;
+        lp.seq_lens = s.seq_lens;
+        lp.h_kv = s.h_kv;
+        lp.units = units;
         lp.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
-        void* lfn = s.head_dim == 64 ? reinterpret_cast<void*>(&window_lse_kernel<64>)
-                                     : reinterpret_cast<void*>(&window_lse_kernel<128>);
+        void* lfn = s.seq_lens ? (s.head_dim == 64 ? reinterpret_cast<void*>(&window_lse_kernel<64, true>)
+                                                   : reinterpret_cast<void*>(&window_lse_kernel<128, true>))
+                               : (s.head_dim == 64 ? reinterpret_cast<void*>(&window_lse_kernel<64, false>)
+                                                   : reinterpret_cast<void*>(&window_lse_kernel<128, false>));
         err = cudaFuncSetAttribute(lfn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.lse_smem_bytes);
         if (err != cudaSuccess) return err;
         void* largs[] = {&lp, &lkmap, &lqmap};
