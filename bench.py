@@ -494,6 +494,11 @@ def extras(step, args):
         out["ragged_lengths"] = {"seq_lens": lens, "us_per_step": round(us, 2), "GB/s": round(rb / (us * 1e-6) / 1e9, 1),
                                  "bytes_per_step": rb}
         del v
+        if step.sel_mode == "carry":   # the same batch with the window LSE computed in the call
+            v = Step(wl, step.budget, step.n_recent, "self", "cuda", share=step, seq_lens=lens_d)
+            v.lse = [None] * wl.layers
+            out["ragged_lengths"]["self_mode_us_per_step"] = round(time_per_step(v.run, n, gs), 2)
+            del v
     out["note"] = "each timed over %d graphed steps outside the headline timed region" % n
     return out
 
