@@ -183,8 +183,9 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
  * bd_draft_attn needs.
  *
  * Arguments and results are those of bd_draft_attn with flags = 0, minus ws and ws_bytes.  The call
- * allocates nothing: its scratch (status word, per-(sequence, KV head) counters and the
- * split-K partials) is a 4 MiB array inside the library's device image, which every GPU
+ * allocates nothing: its scratch (status word and per-(sequence, KV head) counters; the
+ * drafter's split-K partials are merged inside each thread-block cluster) is a 4 MiB
+ * array inside the library's device image, which every GPU
  * that loads the library keeps until the process exits.  A shape whose scratch would not
  * fit returns BD_ERR_WORKSPACE before any launch.
  *   - The first call on a device looks up that array's device address with the device
