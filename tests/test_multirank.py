@@ -65,3 +65,11 @@ def test_reference_arm_prints_on_rank_zero_only():
     assert out.returncode == 0
     line = json.loads(out.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["n_gpus"] == 2 and line["value"] > 0
+    # the reference line's contract: the oracle as cpu_baseline, an e2e without copies
+    assert line["unit"] == "GB/s" and line["higher_is_better"] is True and line["steps"] == 1
+    assert line["config"]["workload"] == "tiny_1k"
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["sample"] and cb["value"] == line["value"]
+    e2e = line["e2e"]
+    assert e2e["value"] == line["value"] and e2e["unit"] == line["unit"]
+    assert e2e["h2d_bytes_per_step"] == 0 and e2e["d2h_bytes_per_step"] == 0
