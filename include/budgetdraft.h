@@ -190,6 +190,8 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
  * fit returns BD_ERR_WORKSPACE before any launch.
  *   - The first call on a device looks up that array's device address with the device
  *     current (cudaGetSymbolAddress); make that first call before any stream capture.
+ *     The address is kept for the life of the process: after cudaDeviceReset on a device
+ *     this entry point has been called on, it must not be called on that device again.
  *   - Every call clears the array's status word and counters on `stream` before its
  *     kernel.  Out-of-range indices are skipped as in bd_draft_attn, but this variant
  *     does not report device-side errors.
@@ -222,7 +224,9 @@ int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_
  *   o_part   fp32 [n_split, rows, d], each row normalised over its own key set;
  *   lse_part fp32 [n_split, rows];
  *   o_out    bf16 [rows, d];  lse_out fp32 [rows] (may be NULL).
- * Constraints: n_split >= 1, rows >= 0 (0 is a no-op), head_dim 64 or 128.
+ * Constraints: 1 <= n_split <= 12288 (the merge weights of a row live in 48 KB of
+ * shared memory; more parts return BD_ERR_UNSUPPORTED), rows >= 0 (0 is a no-op),
+ * head_dim 64 or 128.
  */
 int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows, int head_dim,
                void* o_out, float* lse_out, void* stream);

@@ -275,6 +275,7 @@ int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows
                float* lse_out, void* stream) {
   if (n_split < 1 || rows < 0) return BD_ERR_INVALID_ARG;
   if (head_dim != 64 && head_dim != 128) return BD_ERR_UNSUPPORTED;
+  if (n_split > kCombineMaxSplit) return BD_ERR_UNSUPPORTED;
   if (rows == 0) return BD_OK;
   BD_TRY(check_tensor(o_part, 16));
   BD_TRY(check_tensor(lse_part, 4));

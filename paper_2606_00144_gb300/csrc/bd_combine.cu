@@ -25,7 +25,7 @@ __global__ void __launch_bounds__(kCThreads) combine_kernel(const float* o_part,
 }
 
 int combine_rows_per_block(int n_split) {
-  return std::max(1, std::min(16, 12288 / std::max(1, n_split)));
+  return std::max(1, std::min(16, kCombineMaxSplit / std::max(1, n_split)));
 }
 
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_split, int rows, int head_dim,

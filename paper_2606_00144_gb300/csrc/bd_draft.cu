@@ -348,7 +348,8 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
 // ============================================================================ allocation-free variant
 //
 // bd_draft_attn_static runs the same kernel as bd_draft_attn, but its scratch (status
-// word, per-unit arrival counters, split partials) lives in this file-scope device array
+// word and per-unit arrival counters; the split partials are merged inside each
+// thread-block cluster and need none) lives in this file-scope device array
 // instead of a caller-provided workspace, for callers that cannot allocate device memory.
 // The array is part of the library image: every GPU that loads the library holds it
 // until the process exits.  All calls share it, so calls that overlap on the GPU race.
@@ -360,7 +361,9 @@ size_t draft_static_scratch_bytes() { return kDraftStaticScratchBytes; }
 
 // Device address of g_draft_scratch on the current device.  In host code the symbol is
 // only a host-side stand-in, so the address is looked up once per device, with that
-// device current, and cached.
+// device current, and cached.  A device reset (cudaDeviceReset) unloads the module and
+// leaves the cached address stale: the entry point does not support calls after the
+// reset of a device it has already been called on.
 static cudaError_t draft_scratch_address(void** out) {
   static std::mutex mu;
   static void* addr[256] = {nullptr};

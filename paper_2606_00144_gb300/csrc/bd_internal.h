@@ -94,6 +94,9 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
                           void* ws_region, int* counters, int* status, cudaStream_t stream);
 
 // ---------------------------------------------------------------------------- combine
+// Largest part count of bd_combine: one row's merge weights (n_split floats) must fit the
+// 48 KB of dynamic shared memory a launch gets without opting in.
+constexpr int kCombineMaxSplit = 12288;
 cudaError_t launch_combine(const float* o_part, const float* lse_part, int n_split, int rows,
                            int head_dim, void* o_out, float* lse_out, cudaStream_t stream);
 int combine_rows_per_block(int n_split);

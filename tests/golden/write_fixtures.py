@@ -64,6 +64,23 @@ FIXTURES = {
             {"budget": 12, "chunk": 1, "keep": list(range(12))},
         ],
     },
+    "boundary_example.json": {
+        "cite": "Sec. 3.4 TopKChunks (top floor(B/s) by cumulative attention weight), token level with sink/recent: "
+                "the score of the last middle position the budget admits",
+        "derivation": "t_ctx=10, sink 1, recent 2: middle = positions 1..7 with scores (.5,.9,.6,.7,.3,.55,.1); the "
+                      "sink (10) and recent (8, 7) scores are larger and must not count. Middle scores in descending "
+                      "order: .9,.7,.6,.55,.5,.3,.1. Budget 4 leaves 1 free slot -> tau = .9; budget 5, 2 slots -> "
+                      ".7 (the first excluded score is .6); budget 6, 3 slots -> .6; budget 9, 6 slots -> .3. "
+                      "Budget 3 = sink + recent and budget 2 leave no free slot, budgets 10 and 12 keep everything: "
+                      "nothing is ranked (null).",
+        "t_ctx": 10, "n_sink": 1, "n_recent": 2,
+        "score": [10, 0.5, 0.9, 0.6, 0.7, 0.3, 0.55, 0.1, 8, 7],
+        "cases": [
+            {"budget": 4, "tau": 0.9}, {"budget": 5, "tau": 0.7}, {"budget": 6, "tau": 0.6},
+            {"budget": 9, "tau": 0.3}, {"budget": 3, "tau": None}, {"budget": 2, "tau": None},
+            {"budget": 10, "tau": None}, {"budget": 12, "tau": None},
+        ],
+    },
     "combine_two_halves.json": {
         "cite": "log-sum-exp merge of attention over disjoint key sets (split-K partials)",
         "derivation": "Part A: keys with logits (0, 0) -> lse_A = ln2, o_A = mean of (1,0),(0,1) = (.5,.5). "

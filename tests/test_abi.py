@@ -110,6 +110,7 @@ def test_combine_validation(lib):
     assert f(A, A, 0, 4, 128, A, A, None) == INVALID
     assert f(A, A, 2, -1, 128, A, A, None) == INVALID
     assert f(A, A, 2, 4, 32, A, A, None) == UNSUPPORTED
+    assert f(A, A, 12289, 4, 128, A, A, None) == UNSUPPORTED            # weights beyond 48 KB of smem
     assert f(A, A, 2, 0, 128, A, A, None) == BD_OK                     # empty: no-op
     assert f(A + 4, A, 2, 4, 128, A, A, None) == MISALIGNED
     assert f(A, A, 2, 4, 128, 0, A, None) == INVALID

@@ -70,6 +70,20 @@ def test_golden_selection():
         assert keep.tolist() == case["keep"], case
 
 
+def test_golden_boundary_score():
+    """The tie band of every selection check is centred on this value: the score of the last
+    middle position admitted, not the first one excluded, and nothing when no slot is ranked."""
+    fx = load("boundary_example.json")
+    score = np.array(fx["score"], float)
+    for case in fx["cases"]:
+        tau = oracle.boundary_score(score, fx["t_ctx"], case["budget"], fx["n_sink"], fx["n_recent"])
+        assert tau == case["tau"], case
+        if tau is not None:       # the kept middle is exactly the positions scoring at least tau
+            keep = oracle.select_from_scores(score, fx["t_ctx"], case["budget"], fx["n_sink"], fx["n_recent"])
+            mid = keep[(keep >= fx["n_sink"]) & (keep < fx["t_ctx"] - fx["n_recent"])]
+            assert min(score[mid]) == tau
+
+
 def test_golden_combine():
     fx = load("combine_two_halves.json")
     o, lse = oracle.combine(np.array(fx["o_part"]), np.array(fx["lse_part"]))
@@ -372,6 +386,46 @@ def test_draft_matches_sdpa_over_gathered_rows():
         ref = sdpa_reference(q[0, h][None, None, None], K[0, kv, rows][None, None],
                              V[0, kv, rows][None, None], np.ones((1, rows.size), bool))
         np.testing.assert_allclose(o[0, h], ref[0, 0, 0], atol=1e-13)
+
+
+# ----------------------------------------------------------------------------- one whole step
+
+@pytest.mark.parametrize("budget", [7, 64])
+def test_spec_step_against_independent_routines(budget):
+    """The oracle's whole step (Algorithm 2: sparsify, gamma drafts, verify) against library
+    routines and brute force: the view is the brute-force best subset of the torch-softmax
+    scores, draft pass j is fp64 SDPA over the view plus rows t .. t+j with the j-th draft
+    query, and the verify block is fp64 SDPA with the causal block mask."""
+    rng = np.random.default_rng(18)
+    b, h_q, h_kv, d, t, W, gamma, n_sink, n_recent = 1, 4, 2, 8, 13, 4, 3, 1, 2
+    K, V = rand(rng, b, h_kv, t + gamma + 1, d), rand(rng, b, h_kv, t + gamma + 1, d)
+    qw = rand(rng, b, h_q, W, d)
+    qd = rand(rng, gamma, b, h_q, d)
+    qv = rand(rng, b, h_q, gamma + 1, d)
+    out = oracle.spec_step(K, V, qw, qd, qv, t, budget, n_sink, n_recent)
+    g = h_q // h_kv
+    logits = torch.einsum("bhwd,bhkd->bhwk", torch.from_numpy(qw),
+                          torch.from_numpy(np.repeat(K[:, :, :t], g, axis=1))) / math.sqrt(d)
+    mask = torch.arange(t)[None, :] <= torch.arange(t - W, t)[:, None]
+    score = torch.softmax(logits.masked_fill(~mask, -math.inf), -1).reshape(b, h_kv, g, W, t).sum((2, 3)).numpy()
+    np.testing.assert_allclose(out["score"], score, atol=1e-13)
+    for kv in range(h_kv):
+        keep = brute_force_keep(score[0, kv], t, budget, n_sink, n_recent) if budget < t else list(range(t))
+        assert out["idx"][0, kv, : out["count"][0, kv]].tolist() == keep
+        for j in range(gamma):
+            rows = np.concatenate([np.array(keep, dtype=np.int64), np.arange(t, t + j + 1)])
+            for h in range(kv * g, (kv + 1) * g):
+                ref = sdpa_reference(qd[j, 0, h][None, None, None], K[0, kv, rows][None, None],
+                                     V[0, kv, rows][None, None], np.ones((1, rows.size), bool))
+                np.testing.assert_allclose(out["draft_o"][j, 0, h], ref[0, 0, 0], atol=1e-12)
+                s = K[0, kv, rows] @ qd[j, 0, h] / math.sqrt(d)
+                assert abs(out["draft_lse"][j, 0, h] - logsumexp(s)) < 1e-12
+    Kx = np.repeat(K, g, axis=1)[:, :, : t + gamma + 1]
+    Vx = np.repeat(V, g, axis=1)[:, :, : t + gamma + 1]
+    vmask = np.arange(t + gamma + 1)[None, :] <= (t + np.arange(gamma + 1))[:, None]
+    np.testing.assert_allclose(out["verify_o"], sdpa_reference(qv, Kx, Vx, vmask), atol=1e-12)
+    vlog = np.where(vmask, np.einsum("bhid,bhkd->bhik", qv, Kx) / math.sqrt(d), -np.inf)
+    np.testing.assert_allclose(out["verify_lse"], logsumexp(vlog, axis=-1), atol=1e-12)
 
 
 def test_widen_bf16_bits_exact():

@@ -1,16 +1,20 @@
-"""The allocation-free draft entry point (bd_draft_attn_static) against bd_draft_attn.
+"""The allocation-free draft entry point (bd_draft_attn_static) against the fp64 oracle.
 
 Some callers cannot allocate device memory when they call the library (a plugin handed
 only a stream and tensor pointers, a serving loop whose memory is fixed after start-up).
 bd_draft_attn_static serves them with scratch from the library's own device array.  This
 test calls it through the C ABI twice in a row, with different queries and passes so that
-stale scratch from the first call would show, and checks each result against the
-workspace entry point's on the same inputs, within the parity tolerance.
+stale scratch from the first call would show, and checks each result against
+oracle.draft_attn on the same inputs, within the parity tolerance, and against the
+workspace entry point bd_draft_attn.  The sparse view is a seeded random subset drawn on
+the host, so the oracle's inputs come from the input generators alone.
 """
 
+import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2606_00144_gb300 as bd
 from paper_2606_00144_gb300 import workload as W
 from tests.parity import check_attention, f64
@@ -18,22 +22,36 @@ from tests.parity import check_attention, f64
 pytestmark = pytest.mark.gpu
 
 
+def seeded_view(wl, budget, seed):
+    """Ascending distinct positions of [0, t_ctx) per (sequence, KV head), budget of them."""
+    rng = np.random.default_rng(seed)
+    idx = np.stack([np.sort(rng.choice(wl.t_ctx, budget, replace=False))
+                    for _ in range(wl.batch * wl.h_kv)]).reshape(wl.batch, wl.h_kv, budget)
+    count = np.full((wl.batch, wl.h_kv), budget, dtype=np.int64)
+    return idx, count
+
+
 @pytest.mark.parametrize("budget", [512, 2048])
-def test_draft_attn_static_matches_workspace_entry_point(budget):
+def test_draft_attn_static_matches_oracle(budget):
     """budget 2048: every CTA of a unit's cluster gathers several tiles."""
     bd.build()
     wl = W.WORKLOADS["l8b_16k_b8"]
     inp = W.make_layer(wl, 0, "cuda")
+    idx_h, cnt_h = seeded_view(wl, budget, 7000 + budget)
+    K, V, QD = f64(inp.k_cache), f64(inp.v_cache), f64(inp.q_draft)
     st = bd.SpecStep.for_workload(wl, budget=budget, n_recent=budget // 4)
-    st.select(inp.k_cache, inp.q_win, None)                 # a real sparse view to gather
+    st.idx.copy_(torch.from_numpy(idx_h).int())
+    st.count.copy_(torch.from_numpy(cnt_h).int())
     o = torch.empty(wl.batch, wl.h_q, wl.head_dim, dtype=torch.bfloat16, device="cuda")
     lse = torch.empty(wl.batch, wl.h_q, device="cuda")
     for j in (wl.gamma - 1, 0):                              # two calls in a row
-        st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
         bd.bd_draft_attn_static(st.shape, inp.q_draft[j], inp.k_cache, inp.v_cache, st.idx, st.count,
                                 st.budget, j, o, lse)
+        st.draft(j, inp.q_draft[j], inp.k_cache, inp.v_cache)
         torch.cuda.synchronize()
-        check_attention(o, lse, f64(st.draft_o[j]), f64(st.draft_lse[j]), f"static draft B={budget} j={j}")
+        o_ref, l_ref = oracle.draft_attn(QD[j], K, V, idx_h, cnt_h, wl.t_ctx, j)
+        check_attention(o, lse, o_ref, l_ref, f"static draft B={budget} j={j}")
+        check_attention(o, lse, f64(st.draft_o[j]), f64(st.draft_lse[j]), f"static vs workspace B={budget} j={j}")
     assert st.ws.status() == 0
 
 
