@@ -253,6 +253,10 @@ def timed_replays(graphs, world):
     torch.cuda.synchronize()
     t0 = torch.cuda.Event(enable_timing=True)
     t1 = torch.cuda.Event(enable_timing=True)
+    # the GPU idles for about a millisecond ahead of the start event, so that the host's launch
+    # of the first graph (and its one-time upload to the device) completes before the timed
+    # region opens: the events then bracket the steps' kernels alone
+    torch.cuda._sleep(1 << 21)
     t0.record()
     for g in graphs:
         g.replay()
@@ -363,12 +367,29 @@ def gpu_arm(args):
         "gpu_launches": step.launches_per_step() * args.steps,
         "clocks": clocks,
     }
-    if not args.no_e2e:
-        line["e2e"] = e2e_measure(step, args, world, layer_bytes["total"])
-    if world == 1 and not args.no_extras:
-        line["extras"] = extras(step, args)
+    # the oracle's processes start here (spawned: they import while the GPU lines below run)
+    pool = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, budget, n_recent, args.sel_mode, budget_s=args.cpu_seconds)
+        pool = OraclePool(min(len(os.sched_getaffinity(0)), wl.batch * wl.h_kv * wl.layers))
+    try:
+        if not args.no_e2e:
+            line["e2e"] = e2e_measure(step, args, world, layer_bytes["total"])
+        if world == 1 and not args.no_extras:
+            line["extras"] = extras(step, args)
+            line["extras"]["configs"] = config_table(step, args, us, peak)
+        if pool is not None:
+            line["cpu_baseline"] = cpu_baseline(wl, budget, n_recent, args.sel_mode, args.cpu_seconds, pool)
+            for name, row in line.get("extras", {}).get("configs", {}).items():
+                cw = W.WORKLOADS[name]
+                secs, n_unit, _ = oracle_step(pool, cw, cw.budget, cw.n_recent, "carry", layers=[0])
+                row["cpu_oracle"] = {"us_per_step": round(1e6 * secs, 1), "cores": pool.n,
+                                     "GB/s": round(row["bytes_per_step"] / secs / 1e9, 4),
+                                     "ratio_gpu_vs_oracle": round(1e6 * secs / row["us_per_step"], 1),
+                                     "sample": "one pass over every unit of layer 0" +
+                                               (f", extrapolated x{cw.layers} to all layers" if cw.layers > 1 else "")}
+    finally:
+        if pool is not None:
+            pool.close()
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
@@ -503,6 +524,36 @@ def extras(step, args):
     return out
 
 
+CONFIGS = ("tiny_1k", "l8b_4k", "l8b_8k_b4", "l8b_16k_b8", "l8b_32L_16k_b16")
+
+
+def config_table(head, args, head_us, peak):
+    """Every evaluation workload at its own budget, carry mode, graphed steps: µs per step,
+    tokens verified per second (batch x (gamma + 1) per step), algorithmic bytes and their
+    rate against 8 TB/s and the measured HBM peak.  The headline workload's row is the
+    headline measurement itself."""
+    rows = {}
+    for name in CONFIGS:
+        wl = W.WORKLOADS[name]
+        if name == head.wl.name and head.budget == wl.budget and head.sel_mode == "carry":
+            us, n = head_us, args.steps
+        else:
+            st = Step(wl, wl.budget, wl.n_recent, "carry", "cuda")
+            n = args.extra_steps if wl.layers == 1 else max(20, args.extra_steps // 25)
+            us = time_per_step(st.run, n, args.graph_steps if wl.layers == 1 else 5)
+            del st
+            torch.cuda.empty_cache()
+        b = step_bytes(wl, wl.budget, wl.n_recent, "carry")["total"] * wl.layers
+        gbs = b / (us * 1e-6) / 1e9
+        rows[name] = {"layers": wl.layers, "batch": wl.batch, "t_ctx": wl.t_ctx, "budget": wl.budget,
+                      "n_sink": wl.n_sink, "n_recent": wl.n_recent, "gamma": wl.gamma, "steps_timed": n,
+                      "us_per_step": round(us, 2),
+                      "tokens_verified_per_s": round(wl.batch * (wl.gamma + 1) / (us * 1e-6), 1),
+                      "bytes_per_step": b, "GB/s": round(gbs, 1), "pct_of_8tbs": round(100 * gbs / NOMINAL_HBM_GBS, 1),
+                      "frac_of_measured_hbm": round(gbs / peak, 3)}
+    return rows
+
+
 def e2e_measure(step, args, world, bytes_per_step):
     """The same steps driven from pinned host buffers through HostStepIO (the package's
     host-buffer API): every step copies its inputs host->device and its results back,
@@ -584,85 +635,134 @@ def measured_hbm_peak():
 
 # ----------------------------------------------------------------------------- oracle timing
 
-class OraclePieces:
-    """The oracle's step, one (sequence, KV head) unit at a time, in pieces:
-    selection (carried LSE), the gamma draft passes, the verify block."""
-
-    def __init__(self, wl, budget, n_recent, sel_mode):
-        import oracle
-        self.oracle = oracle
-        self.wl, self.budget, self.n_recent, self.sel_mode = wl, budget, n_recent, sel_mode
-        self.row = wl.head_dim * 2
-        self.units = [(b, kv) for b in range(wl.batch) for kv in range(wl.h_kv)]
-        self.seq_cache = {}
-        self.next_unit = 0
-        self.queue = []
-
-    def _unit(self, b, kv):
-        if b not in self.seq_cache:
-            self.seq_cache.clear()
-            one = dataclasses.replace(self.wl, batch=1)
-            inp = W.make_layer(one, 0, "cpu", first_seq=b)      # sequence b's own seed
-            f = lambda t: t.to(torch.float64).numpy()
-            self.seq_cache[b] = tuple(map(f, (inp.k_cache, inp.v_cache, inp.q_win, inp.q_draft, inp.q_verify)))
-        K, V, QW, QD, QV = self.seq_cache[b]
-        g = self.wl.group
-        hs = slice(kv * g, (kv + 1) * g)
-        return dict(K=K[:, kv:kv + 1], V=V[:, kv:kv + 1], QW=QW[:, hs], QD=QD[:, :, hs], QV=QV[:, hs])
-
-    def _refill(self):
-        b, kv = self.units[self.next_unit % len(self.units)]
-        self.next_unit += 1
-        u = self._unit(b, kv)
-        o = self.oracle
-        wl = self.wl
-        lse = None if self.sel_mode == "self" else o.window_lse(u["QW"], u["K"], wl.t_ctx)   # carried state
-        state = {}
-        sel_bytes = 0 if self.budget >= wl.t_ctx else (wl.t_ctx - wl.n_sink - self.n_recent) * self.row
-        if self.sel_mode == "self" and self.budget < wl.t_ctx:
-            sel_bytes += wl.t_ctx * self.row
-
-        def select():
-            idx, cnt, _ = o.select_budget(u["QW"], u["K"], wl.t_ctx, self.budget, wl.n_sink, self.n_recent,
-                                          1, lse)
-            state["idx"], state["cnt"] = idx, cnt
-
-        draft_bytes = (min(self.budget, wl.t_ctx) + wl.gamma) * 2 * self.row / wl.gamma
-
-        def draft(j):
-            return lambda: o.draft_attn(u["QD"][j], u["K"], u["V"], state["idx"], state["cnt"], wl.t_ctx, j)
-
-        def verify():
-            o.verify_attn(u["QV"], u["K"], u["V"], wl.t_ctx)
-
-        self.queue = [(select, sel_bytes)] + [(draft(j), draft_bytes) for j in range(wl.gamma)] + \
-                     [(verify, (wl.t_ctx + wl.gamma + 1) * 2 * self.row)]
-
-    def run_piece(self):
-        if not self.queue:
-            self._refill()
-        fn, nbytes = self.queue.pop(0)
-        t0 = time.perf_counter()
-        fn()
-        return time.perf_counter() - t0, nbytes
+def unit_bytes(wl, budget, n_recent, sel_mode, n_sink=None):
+    """Algorithmic bytes of one (sequence, KV head) unit's step."""
+    units = wl.batch * wl.h_kv
+    return step_bytes(wl, budget, n_recent, sel_mode, n_sink)["total"] / units
 
 
-def cpu_baseline(wl, budget, n_recent, sel_mode, budget_s=12.0):
-    pieces = OraclePieces(wl, budget, n_recent, sel_mode)
-    secs, nbytes, n = 0.0, 0.0, 0
-    per_unit = 2 + wl.gamma
-    t_start = time.perf_counter()
-    while (secs < budget_s or n % per_unit) and time.perf_counter() - t_start < 4 * budget_s:
-        s, b = pieces.run_piece()
-        secs += s
-        nbytes += b
-        n += 1
-    units = n // per_unit
-    return {"value": round(nbytes / secs / 1e9, 4), "unit": "GB/s",
-            "cores": int(os.environ.get("OMP_NUM_THREADS", "1")), "kind": "oracle",
-            "sample": f"{units} (sequence, KV head) unit-steps of one layer, cycling over its "
-                      f"{wl.batch * wl.h_kv} units; each = selection with the carried LSE, {wl.gamma} drafts and "
-                      f"the verify block, numpy fp64; {secs:.1f} s of oracle time"}
+def _draw_sequence(wl, layer, b):
+    """Sequence b of `layer` drawn on the host by the workload recipe, as fp64 arrays."""
+    one = dataclasses.replace(wl, batch=1)
+    inp = W.make_layer(one, layer, "cpu", first_seq=b)
+    f = lambda t: t.to(torch.float64).numpy()
+    return tuple(map(f, (inp.k_cache, inp.v_cache, inp.q_win, inp.q_draft, inp.q_verify)))
+
+
+def _oracle_worker(rank, tasks, results, barrier):
+    """One host core (single-threaded BLAS): per task, draws its (layer, sequence, KV head)
+    units' inputs and the carried window LSE (not timed), then for every pass waits for the
+    other workers and runs the oracle's whole step on each of its units: the selection, the
+    gamma draft passes over the oracle's own view, the verify block."""
+    import oracle
+    while True:
+        task = tasks.get()
+        if task is None:
+            return
+        wl, budget, n_recent, sel_mode, units, passes = task
+        g = wl.group
+        data, seq = [], {}
+        for (l, b, kv) in units:
+            if (l, b) not in seq:
+                seq.clear()
+                seq[(l, b)] = _draw_sequence(wl, l, b)
+            K, V, QW, QD, QV = seq[(l, b)]
+            hs = slice(kv * g, (kv + 1) * g)
+            u = dict(K=K[:, kv:kv + 1].copy(), V=V[:, kv:kv + 1].copy(), QW=QW[:, hs].copy(),
+                     QD=QD[:, :, hs].copy(), QV=QV[:, hs].copy())
+            u["lse"] = oracle.window_lse(u["QW"], u["K"], wl.t_ctx) if sel_mode == "carry" else None
+            data.append(u)
+        seq.clear()
+        out = []
+        for _ in range(passes):
+            barrier.wait()
+            t0 = time.monotonic()
+            for u in data:
+                oracle.spec_step(u["K"], u["V"], u["QW"], u["QD"], u["QV"], wl.t_ctx, budget, wl.n_sink, n_recent,
+                                 lse_win=u["lse"])
+            out.append((t0, time.monotonic(), len(data)))
+        results.put((rank, out))
+
+
+class OraclePool:
+    """The fp64 oracle on the host cores: one spawned process per core of
+    os.sched_getaffinity(0), each with single-threaded BLAS, over independent
+    (layer, sequence, KV head) units.  A pass runs every unit of the sample once, all
+    workers starting together; its time is the span from the first start to the last end."""
+
+    def __init__(self, n_workers=None):
+        import multiprocessing as mp
+        self.n = max(1, n_workers or len(os.sched_getaffinity(0)))
+        ctx = mp.get_context("spawn")
+        self.barrier = ctx.Barrier(self.n)
+        self.tasks = [ctx.Queue() for _ in range(self.n)]
+        self.results = ctx.Queue()
+        saved = {v: os.environ.get(v) for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS")}
+        os.environ.update({v: "1" for v in saved})            # the children inherit one BLAS thread each
+        try:
+            self.procs = [ctx.Process(target=_oracle_worker, args=(i, self.tasks[i], self.results, self.barrier),
+                                      daemon=True) for i in range(self.n)]
+            for p in self.procs:
+                p.start()
+        finally:
+            for v, x in saved.items():
+                if x is None:
+                    os.environ.pop(v, None)
+                else:
+                    os.environ[v] = x
+
+    def run(self, wl, budget, n_recent, sel_mode, units, passes):
+        """Runs `passes` passes over `units` [(layer, b, kv)]; returns [(seconds, unit_steps)] per pass."""
+        per = (len(units) + self.n - 1) // self.n
+        for i in range(self.n):
+            self.tasks[i].put((wl, budget, n_recent, sel_mode, units[i * per:(i + 1) * per], passes))
+        res = [self.results.get(timeout=3600) for _ in range(self.n)]
+        spans = []
+        for p in range(passes):
+            starts = [r[1][p][0] for r in res]
+            ends = [r[1][p][1] for r in res]
+            spans.append((max(ends) - min(starts), sum(r[1][p][2] for r in res)))
+        return spans
+
+    def close(self):
+        for q in self.tasks:
+            q.put(None)
+        for p in self.procs:
+            p.join(timeout=30)
+
+
+def layer_units(wl, layers=None):
+    layers = range(wl.layers) if layers is None else layers
+    return [(l, b, kv) for l in layers for b in range(wl.batch) for kv in range(wl.h_kv)]
+
+
+def oracle_step(pool, wl, budget, n_recent, sel_mode, layers=None, passes=1):
+    """The oracle's time for one whole step of the workload (every unit of the given layers,
+    scaled to all layers when only a sample of them ran)."""
+    units = layer_units(wl, layers)
+    spans = pool.run(wl, budget, n_recent, sel_mode, units, passes)
+    secs = sum(s for s, _ in spans) / len(spans)
+    scale = wl.layers / (len(units) / (wl.batch * wl.h_kv))
+    return secs * scale, len(units) * len(spans), secs
+
+
+def cpu_baseline(wl, budget, n_recent, sel_mode, budget_s=12.0, pool=None):
+    own = pool is None
+    pool = pool or OraclePool(min(len(os.sched_getaffinity(0)), wl.batch * wl.h_kv))
+    try:
+        # one pass to size the sample, then enough whole-layer passes for about budget_s of CPU work
+        s1, _, _ = oracle_step(pool, wl, budget, n_recent, sel_mode, layers=[0])
+        passes = max(1, min(50, int(budget_s / max(s1 * pool.n, 1e-3))))
+        secs, n_unit, _ = oracle_step(pool, wl, budget, n_recent, sel_mode, layers=[0], passes=passes)
+    finally:
+        if own:
+            pool.close()
+    step_b = step_bytes(wl, budget, n_recent, sel_mode)["total"]
+    return {"value": round(step_b / secs / 1e9, 4), "unit": "GB/s", "cores": pool.n, "kind": "oracle",
+            "us_per_step": round(1e6 * secs, 1),
+            "sample": f"{passes} whole steps of one layer ({wl.batch * wl.h_kv} (sequence, KV head) units, each the "
+                      f"selection with the carried window LSE, {wl.gamma} draft passes and the verify block), the "
+                      f"units spread over {pool.n} single-threaded processes; numpy fp64"}
 
 
 def reference_arm(args):
@@ -670,31 +770,32 @@ def reference_arm(args):
     if rank != 0:
         return
     wl = resolve_workload(args)
-    pieces = OraclePieces(wl, wl.budget, wl.n_recent, args.sel_mode)
-    for _ in range(args.warmup):
-        pieces.run_piece()
-    secs, nbytes = 0.0, 0.0
-    for _ in range(args.steps):
-        s, b = pieces.run_piece()
-        secs += s
-        nbytes += b
-    value = nbytes / secs / 1e9
-    ms_per_step = 1e3 * secs / args.steps
-    cores = int(os.environ.get("OMP_NUM_THREADS", "1"))
-    sample = (f"each step = one piece of one (sequence, KV head) unit's step (selection with carried LSE, one of "
-              f"{wl.gamma} draft passes, or the verify block), round robin; fp64 numpy oracle")
+    units = layer_units(wl, [0])
+    pool = OraclePool(min(len(os.sched_getaffinity(0)), len(units)))
+    try:
+        spans = pool.run(wl, wl.budget, wl.n_recent, args.sel_mode, units, args.warmup + args.steps)
+    finally:
+        pool.close()
+    secs = sum(s for s, _ in spans[args.warmup:])
+    step_b = step_bytes(wl, wl.budget, wl.n_recent, args.sel_mode)["total"]
+    value = step_b * args.steps / secs / 1e9
+    sample = (f"each step = one whole step of one layer of the workload ({len(units)} (sequence, KV head) units: "
+              f"selection with the carried window LSE, {wl.gamma} draft passes, the verify block) on "
+              f"{pool.n} single-threaded processes; fp64 numpy oracle")
     line = {
         "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s", "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 4),
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(1e3 * secs / args.steps, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
         "data": "synthetic (same recipe as the GPU arm, drawn on the host)",
         "config": {"workload": wl.name, "layers": wl.layers, "batch": wl.batch, "h_q": wl.h_q, "h_kv": wl.h_kv,
                    "head_dim": wl.head_dim, "t_ctx": wl.t_ctx, "budget": wl.budget, "n_sink": wl.n_sink,
                    "n_recent": wl.n_recent, "window": wl.window, "gamma": wl.gamma, "sel_mode": args.sel_mode},
-        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": cores, "kind": "oracle",
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": pool.n, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
+    if wl.layers > 1:
+        line["note"] = f"one layer of {wl.layers} per step"
     print(json.dumps(line), flush=True)
 
 

@@ -1,9 +1,13 @@
 // Warp-level attention over 16-key sub-tiles on mma.sync (shared by the verify and draft
 // kernels).  Keys sit on the M side: S^T = K Q^T with the query rows on N (8*NT columns),
-// so a GQA group x block of query rows fills n8 tiles without padding to 16.  P^T is
-// rounded to bf16, each 8x8 block transposed in registers with movmatrix to become the B
-// operand, and O^T = V^T P^T accumulates with V^T read by ldmatrix.trans.  Softmax state
-// (running max m and sum l per query column) lives in the exp2 domain.
+// so a GQA group x block of query rows fills n8 tiles without padding to 16.  P^T (fp32)
+// is split into two bf16 terms, P = P_hi + P_lo with P_hi = bf16(P) and P_lo = bf16(P - P_hi),
+// each 8x8 block transposed in registers with movmatrix to become the B operand, and
+// O^T = V^T P_hi^T + V^T P_lo^T accumulates with V^T read by ldmatrix.trans.  The pair
+// carries P to about 2^-17 relative, so the weights of O keep nearly fp32 precision: with
+// P rounded to one bf16 alone (2^-9), an output element of 1e-3 over a few hundred keys
+// could be off by more than 1e-5.  Softmax state (running max m and sum l per query column)
+// lives in the exp2 domain.
 //
 // K/V sub-tiles are read from shared memory in the TMA SWIZZLE_128B layout (sw128_offset).
 #pragma once
@@ -111,11 +115,16 @@ struct WarpAttn {
             o[mt][nt][3] *= alpha[nt][1];
           }
       }
-      uint32_t bp[NT][2];
+      uint32_t bp[NT][2], bl[NT][2];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        bp[nt][0] = movmatrix_trans(pack_bf16x2(s[nt][0], s[nt][1]));
-        bp[nt][1] = movmatrix_trans(pack_bf16x2(s[nt][2], s[nt][3]));
+        uint32_t h0, l0, h1, l1;
+        split_bf16x2(s[nt][0], s[nt][1], h0, l0);
+        split_bf16x2(s[nt][2], s[nt][3], h1, l1);
+        bp[nt][0] = movmatrix_trans(h0);
+        bp[nt][1] = movmatrix_trans(h1);
+        bl[nt][0] = movmatrix_trans(l0);
+        bl[nt][1] = movmatrix_trans(l1);
       }
 #pragma unroll
       for (int mt = 0; mt < KS; ++mt) {
@@ -123,7 +132,10 @@ struct WarpAttn {
         ldmatrix_x4_trans(a, vbase + sw128_offset(kb + (lane & 7) + 8 * (lane >> 4), 16 * mt + 8 * ((lane >> 3) & 1),
                                                   half_bytes));
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) mma_16816(o[mt][nt], a, bp[nt][0], bp[nt][1]);
+        for (int nt = 0; nt < NT; ++nt) {
+          mma_16816(o[mt][nt], a, bp[nt][0], bp[nt][1]);
+          mma_16816(o[mt][nt], a, bl[nt][0], bl[nt][1]);
+        }
       }
     }
   }

@@ -87,6 +87,15 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Two-term bf16 form of a pair of floats: head = bf16x2(x, y) rounded to nearest, tail =
+// bf16x2 of what the rounding left over, so that head + tail carries about 16 bits of each
+// value's significand (x in the low halves, y in the high halves).
+__device__ __forceinline__ void split_bf16x2(float x, float y, uint32_t& head, uint32_t& tail) {
+  head = pack_bf16x2(x, y);
+  const float hx = __uint_as_float(head << 16), hy = __uint_as_float(head & 0xffff0000u);
+  tail = pack_bf16x2(x - hx, y - hy);
+}
+
 // Every wait in these kernels gives up after this long (or this many polls) and records
 // BD_ERR_TIMEOUT in the workspace status word, so a logic error can never hang the GPU.
 constexpr uint64_t kWaitLimitNs = 2000000000ull;   // 2 s

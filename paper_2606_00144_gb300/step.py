@@ -73,11 +73,20 @@ class SpecStep:
 
     def window_lse(self, k_cache, q_win, out=None, stream=None):
         """LSE of the window queries over their causal prefixes, computed by the verify
-        kernel (what a previous verify / prefill step leaves behind for carry mode)."""
+        kernel (what a previous verify / prefill step leaves behind for carry mode).
+
+        The window rows form a verify block that starts W positions before the context's
+        end.  With per-sequence lengths, sequence b's rows sit at seq_lens[b] - W ..
+        seq_lens[b] - 1, so every length must exceed the window W."""
+        lens = None
         if self.seq_lens is not None:
-            raise NotImplementedError("window_lse with per-sequence lengths: use bd_select_budget's self mode")
+            ts = torch.cuda.ExternalStream(stream) if isinstance(stream, int) else \
+                (stream or torch.cuda.current_stream())
+            with torch.cuda.stream(ts):
+                lens = torch.sub(self.seq_lens, self.window)          # where each window block starts
+            lens.record_stream(ts)
         sh = B.make_shape(self.shape.batch, self.shape.h_q, self.shape.h_kv, self.shape.head_dim,
-                          self.shape.t_ctx - self.window, self.shape.t_cap)
+                          self.shape.t_ctx - self.window, self.shape.t_cap, lens)
         if out is None:
             out = torch.empty(self.shape.batch, self.shape.h_q, self.window, dtype=torch.float32,
                               device=k_cache.device)

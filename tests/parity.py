@@ -54,7 +54,8 @@ def check_attention(o_gpu, lse_gpu, o_ref, lse_ref, what=""):
         lr = np.asarray(lse_ref, dtype=np.float64).reshape(-1)
         both_inf = np.isneginf(lg) & np.isneginf(lr)
         assert np.array_equal(np.isneginf(lg), np.isneginf(lr)), f"{what}: -inf lse mismatch"
-        lerr = np.abs(np.where(both_inf, 0.0, lg - lr))
+        lerr = np.zeros_like(lg)
+        lerr[~both_inf] = np.abs(lg[~both_inf] - lr[~both_inf])
         assert lerr.max() <= LSE_ATOL, f"{what}: lse err {lerr.max():.3e}"
         out["lse_abs"] = float(lerr.max())
     return out

@@ -289,37 +289,34 @@ def test_combine_standalone():
 
 
 def test_combine_merges_disjoint_draft_views():
-    # attention over idx split into two disjoint halves, merged by bd_combine == attention over all
+    """Draft attention over two disjoint halves of a view, merged by bd_combine, equals draft
+    attention over the whole view.  The halves' results (the parts a split-K caller hands to
+    bd_combine, in its fp32 input type) come from the oracle's draft pass; the GPU's own
+    split-K drafts are checked in every draft parity case."""
     wl = W.tiny_workload(batch=1, h_q=8, h_kv=2, head_dim=128, t_ctx=900, budget=128)
     inp = W.make_layer(wl, 0, "cuda")
     h = host(inp)
     rng = np.random.default_rng(9)
     full = np.stack([np.sort(rng.choice(900, 128, replace=False)) for _ in range(2)])[None]
-    st = bd.SpecStep.for_workload(wl)
     parts_o, parts_l = [], []
     for half in (slice(0, 64), slice(64, 128)):
         sub = np.full((1, 2, 128), -1)
         sub[..., :64] = full[..., half]
-        st.idx.copy_(torch.from_numpy(sub).int())
-        st.count.fill_(64)
-        st.draft(0, inp.q_draft[0], inp.k_cache, inp.v_cache)
-        torch.cuda.synchronize()
-        parts_o.append(st.draft_o[0].float().reshape(-1, 128).clone())
-        parts_l.append(st.draft_lse[0].reshape(-1).clone())
-    # the tail row t_ctx is in both parts: remove it from the second by merging against it once
-    o_part = torch.stack(parts_o)
-    l_part = torch.stack(parts_l)
+        o, l = oracle.draft_attn(h["QD"][0], h["K"], h["V"], sub, np.full((1, 2), 64), 900, 0)
+        parts_o.append(o.reshape(-1, 128))
+        parts_l.append(l.reshape(-1))
+    o_part = torch.from_numpy(np.stack(parts_o)).float().cuda()
+    l_part = torch.from_numpy(np.stack(parts_l)).float().cuda()
     out = torch.empty(8, 128, dtype=torch.bfloat16, device="cuda")
     lse = torch.empty(8, device="cuda")
     bd.bd_combine(o_part, l_part, 2, 8, 128, out, lse)
-    rows0 = np.concatenate([full[0, :, :64], np.full((2, 1), 900)], axis=1)
-    rows1 = np.concatenate([full[0, :, 64:], np.full((2, 1), 900)], axis=1)
+    # each part also attended to the drafted row t_ctx: the union counts it twice
+    both = np.concatenate([full[0], np.full((2, 2), 900)], axis=1)
     o_ref = np.zeros((8, 128))
     l_ref = np.zeros(8)
     for hh in range(8):
         kv = hh // 4
-        rows = np.concatenate([rows0[kv], rows1[kv]])       # the tail row counted twice, like the parts
-        o_ref[hh], l_ref[hh] = oracle.attention(h["QD"][0, 0, hh], h["K"][0, kv, rows], h["V"][0, kv, rows],
+        o_ref[hh], l_ref[hh] = oracle.attention(h["QD"][0, 0, hh], h["K"][0, kv, both[kv]], h["V"][0, kv, both[kv]],
                                                 1 / np.sqrt(128))
     torch.cuda.synchronize()
     check_attention(out, lse, o_ref, l_ref, "combine of draft parts")

@@ -94,6 +94,25 @@ def test_ragged_lengths_match_per_sequence_oracle(mode):
     assert ws.status() == 0
 
 
+def test_ragged_window_lse_matches_oracle():
+    """SpecStep.window_lse with per-sequence lengths: each sequence's window rows over its own
+    causal prefix (the carried state a prefill leaves for carry mode)."""
+    lens = [3000, 2433, 1777, 200]
+    b, hq, hkv, d, W = len(lens), 8, 2, 128, 32
+    wl = wk.tiny_workload(batch=b, h_q=hq, h_kv=hkv, head_dim=d, t_ctx=max(lens), budget=256, n_sink=4,
+                         n_recent=64, window=W, gamma=3)
+    inp = wk.make_layer(wl, 0, "cuda")
+    lens_d = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    st = bd.SpecStep(b, hq, hkv, d, wl.t_ctx, wl.t_cap, 256, 4, 64, W, 3, seq_lens=lens_d)
+    lse = st.window_lse(inp.k_cache, inp.q_win)
+    torch.cuda.synchronize()
+    K, QW = f64(inp.k_cache), f64(inp.q_win)
+    for i, t in enumerate(lens):
+        ref = oracle.window_lse(QW[i:i + 1], K[i:i + 1], t)
+        err = np.abs(f64(lse[i:i + 1]) - ref).max()
+        assert err <= 1e-3, f"seq {i} T={t}: window lse err {err:.3e}"
+
+
 def test_ragged_block_rows_land_at_each_sequence_length():
     lens = [50, 37, 64]
     b, hkv, d, n_rows, t_cap = len(lens), 2, 64, 4, 80
