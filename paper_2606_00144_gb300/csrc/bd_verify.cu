@@ -324,11 +324,13 @@ Variant pick_variant(int nq_rows, bool with_v) {
 struct KernelInfo {
   void* fn;
   size_t smem;
+  size_t merge_floats;   // the staging area a unit's last CTA merges the segments' partials in
 };
 
 template <int D, int NT, int WQ, bool WITH_V>
 KernelInfo info() {
-  return {reinterpret_cast<void*>(&verify_kernel<D, NT, WQ, WITH_V>), VerifySmem<D, NT, WQ, WITH_V>::kTotal};
+  return {reinterpret_cast<void*>(&verify_kernel<D, NT, WQ, WITH_V>), VerifySmem<D, NT, WQ, WITH_V>::kTotal,
+          VerifySmem<D, NT, WQ, WITH_V>::kMerge / 4};
 }
 
 KernelInfo select_kernel(int d, int nt, int wq, bool with_v) {
@@ -339,7 +341,7 @@ KernelInfo select_kernel(int d, int nt, int wq, bool with_v) {
   BD_VK(64, 4, 1, false) BD_VK(64, 4, 2, false) BD_VK(64, 4, 4, false)
   BD_VK(128, 4, 1, false) BD_VK(128, 4, 2, false) BD_VK(128, 4, 4, false)
 #undef BD_VK
-  return {nullptr, 0};
+  return {nullptr, 0, 0};
 }
 
 // Resident CTAs per SM of a kernel (cached per kernel and device).
@@ -390,6 +392,14 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   if (vtotal >= (1L << 31)) return false;
   long vtpc = (vtotal + ctas - 1) / ctas;
   vtpc = std::max<long>(vtpc, (tpu + a + kVMaxSeg - 2) / (kVMaxSeg - 1));   // <= kVMaxSeg segments
+  // The unit's last CTA merges its segments in one round trip while they fit its staging
+  // area; beyond that the merge reads every part of every output element from L2 in turn,
+  // which costs far more than the streaming balance gains (a 4K context at batch 1: 16
+  // segments per unit, 24 us).  So, where the area holds two parts or more, a unit spans at
+  // most that many CTAs: a span of L tiles cut into ranges of v touches at most
+  // ceil((L - 1) / v) + 1 of them.
+  const long cap = with_v ? (long)(k.merge_floats / ((size_t)nq_rows * s.head_dim)) : 0;
+  if (cap >= 2) vtpc = std::max<long>(vtpc, (tpu + a - 1 + cap - 2) / (cap - 1));
   plan->seg_cost = a;
   plan->tiles_per_cta = (int)vtpc;
   plan->total_tiles = (int)total;
