@@ -39,6 +39,7 @@ struct VerifyPlan {
   int stages;
   size_t smem_bytes;
   bool with_v;
+  bool wide;            // more segments per unit than one staged merge round holds
 };
 bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan);
 size_t verify_partials_bytes(const bd_shape& s, const VerifyPlan& plan);

@@ -38,6 +38,7 @@ struct VerifyParams {
   float* o_part;       // [units][max_seg][nq_rows][D]
   float* lse_part;     // [units][max_seg][nq_rows]
   int* counters;       // [units]
+  int* nseg;           // [units] segments of each unit (wide plans: read by verify_merge_kernel)
   int* status;
   const int32_t* seq_lens;  // per-sequence context lengths [batch] or null (all t_ctx)
   int h_kv;
@@ -95,7 +96,13 @@ struct VerifySmem {
   static constexpr size_t kTotal = 1024 + 1024 + kStages + kMerge + kWeights;
 };
 
-template <int D, int NT, int WQ, bool WITH_V>
+// WIDE: the instance for plans whose units span more CTAs than the last one can merge in a
+// single staged round trip (small and mid-size batches).  Every CTA only writes its
+// segment's partial, the unit's first CTA its segment count, and verify_merge_kernel,
+// launched right after, merges them with the whole GPU: a last-CTA merge of ten to twenty
+// parts cost 10-16 us at the end of the kernel.  A separate instance, so that the common
+// case's code (and register allocation) stays as it is.
+template <int D, int NT, int WQ, bool WITH_V, bool WIDE>
 __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
                                                            const __grid_constant__ CUtensorMap kmap,
                                                            const __grid_constant__ CUtensorMap vmap) {
@@ -270,9 +277,15 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     const int c_last = map.owner(unit, map.tiles(unit) - 1);
     const int n_seg = c_last - c_first + 1;
     const size_t row0 = (size_t)unit * nq;
+    if (WIDE && c == c_first && tid == 0) p.nseg[unit] = n_seg;
     if (n_seg == 1) {
       merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, nq, p.lse ? p.lse + row0 : nullptr,
                                            WITH_V ? static_cast<void*>(p.o + row0 * D) : nullptr, true, tid, NCT, 1);
+    } else if constexpr (WIDE) {
+      const size_t slot = (size_t)unit * p.max_seg + (c - c_first);
+      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, nq, p.lse_part + slot * nq,
+                                           WITH_V ? static_cast<void*>(p.o_part + slot * nq * D) : nullptr, false,
+                                           tid, NCT, 1);
     } else {
       const size_t slot = (size_t)unit * p.max_seg + (c - c_first);
       merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, nq, p.lse_part + slot * nq,
@@ -296,6 +309,82 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     if (tid == 0) last_flag[1] = *abort_flag;
     named_bar(1, NCT);
     if (last_flag[1]) break;
+  }
+}
+
+// Merge of the segments' partials for the wide plans: one CTA per (unit, output row); a
+// unit whose segment count is 1 was written by the verify kernel itself.  Thread t takes
+// four adjacent columns (t % (D/4)) of the segments s = t / (D/4) (mod 128 / (D/4)), so
+// every part of the row is requested at once: the lse values, then the rows, two round
+// trips to L2 in all; the groups' sums meet in shared memory.
+template <int D>
+__global__ void __launch_bounds__(128) verify_merge_kernel(const float* o_part, const float* lse_part,
+                                                           const int* nseg, int max_seg, int nq,
+                                                           __nv_bfloat16* o, float* lse) {
+  constexpr int Q = D / 4;                 // column quads per row
+  constexpr int NG = 128 / Q;              // segment groups
+  constexpr int PER = (kVMaxSeg + NG - 1) / NG;
+  grid_dependency_wait();
+  allow_dependent_launch();
+  __shared__ float w[kVMaxSeg];
+  __shared__ float4 part[NG][Q];
+  const int unit = blockIdx.x, r = blockIdx.y, tid = threadIdx.x;
+  const int n = min(__ldcg(nseg + unit), kVMaxSeg);
+  if (n <= 1) return;
+  const size_t base = (size_t)unit * max_seg;
+  if (tid < 32) {
+    const float l0 = tid < n ? __ldcg(lse_part + (base + tid) * nq + r) : -INFINITY;
+    const float l1 = tid + 32 < n ? __ldcg(lse_part + (base + tid + 32) * nq + r) : -INFINITY;
+    float mx = fmaxf(l0, l1);
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, off));
+    const float e0 = mx == -INFINITY ? 0.f : fast_exp2((l0 - mx) * kLog2e);
+    const float e1 = mx == -INFINITY ? 0.f : fast_exp2((l1 - mx) * kLog2e);
+    float tot = e0 + e1;
+#pragma unroll
+    for (int off = 16; off > 0; off >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, off);
+    const float inv = tot > 0.f ? 1.f / tot : 0.f;
+    if (tid < n) w[tid] = e0 * inv;
+    if (tid + 32 < n) w[tid + 32] = e1 * inv;
+    if (tid == 0 && lse) lse[(size_t)unit * nq + r] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
+  }
+  if (o == nullptr) return;
+  const int q = tid % Q, g = tid / Q;
+  float4 v[PER];
+#pragma unroll
+  for (int k = 0; k < PER; ++k) {
+    const int sg = g + NG * k;
+    v[k] = sg < n ? __ldcg(reinterpret_cast<const float4*>(o_part + ((base + sg) * nq + r) * D) + q)
+                  : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  __syncthreads();                                  // the weights
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+  for (int k = 0; k < PER; ++k) {
+    const int sg = g + NG * k;
+    const float wk = sg < n ? w[sg] : 0.f;
+    if (wk != 0.f) {                                // an empty part never enters the sum
+      acc.x += wk * v[k].x;
+      acc.y += wk * v[k].y;
+      acc.z += wk * v[k].z;
+      acc.w += wk * v[k].w;
+    }
+  }
+  part[g][q] = acc;
+  __syncthreads();
+  if (g == 0) {
+#pragma unroll
+    for (int h = 1; h < NG; ++h) {
+      const float4 b = part[h][q];
+      acc.x += b.x;
+      acc.y += b.y;
+      acc.z += b.z;
+      acc.w += b.w;
+    }
+    uint2 packed;
+    packed.x = pack_bf16x2(acc.x, acc.y);
+    packed.y = pack_bf16x2(acc.z, acc.w);
+    *reinterpret_cast<uint2*>(o + ((size_t)unit * nq + r) * D + 4 * q) = packed;
   }
 }
 
@@ -327,19 +416,23 @@ struct KernelInfo {
   size_t merge_floats;   // the staging area a unit's last CTA merges the segments' partials in
 };
 
-template <int D, int NT, int WQ, bool WITH_V>
+template <int D, int NT, int WQ, bool WITH_V, bool WIDE>
 KernelInfo info() {
-  return {reinterpret_cast<void*>(&verify_kernel<D, NT, WQ, WITH_V>), VerifySmem<D, NT, WQ, WITH_V>::kTotal,
+  return {reinterpret_cast<void*>(&verify_kernel<D, NT, WQ, WITH_V, WIDE>), VerifySmem<D, NT, WQ, WITH_V>::kTotal,
           VerifySmem<D, NT, WQ, WITH_V>::kMerge / 4};
 }
 
-KernelInfo select_kernel(int d, int nt, int wq, bool with_v) {
-#define BD_VK(DD, N, W, V) \
-  if (d == DD && nt == N && wq == W && with_v == V) return info<DD, N, W, V>();
-  BD_VK(64, 1, 1, true) BD_VK(64, 3, 1, true) BD_VK(64, 3, 2, true) BD_VK(64, 3, 4, true)
-  BD_VK(128, 1, 1, true) BD_VK(128, 3, 1, true) BD_VK(128, 3, 2, true) BD_VK(128, 3, 4, true)
-  BD_VK(64, 4, 1, false) BD_VK(64, 4, 2, false) BD_VK(64, 4, 4, false)
-  BD_VK(128, 4, 1, false) BD_VK(128, 4, 2, false) BD_VK(128, 4, 4, false)
+KernelInfo select_kernel(int d, int nt, int wq, bool with_v, bool wide) {
+#define BD_VK(DD, N, W, V, X) \
+  if (d == DD && nt == N && wq == W && with_v == V && wide == X) return info<DD, N, W, V, X>();
+  BD_VK(64, 1, 1, true, false) BD_VK(64, 3, 1, true, false) BD_VK(64, 3, 2, true, false) BD_VK(64, 3, 4, true, false)
+  BD_VK(128, 1, 1, true, false) BD_VK(128, 3, 1, true, false) BD_VK(128, 3, 2, true, false)
+  BD_VK(128, 3, 4, true, false)
+  BD_VK(64, 1, 1, true, true) BD_VK(64, 3, 1, true, true) BD_VK(64, 3, 2, true, true) BD_VK(64, 3, 4, true, true)
+  BD_VK(128, 1, 1, true, true) BD_VK(128, 3, 1, true, true) BD_VK(128, 3, 2, true, true)
+  BD_VK(128, 3, 4, true, true)
+  BD_VK(64, 4, 1, false, false) BD_VK(64, 4, 2, false, false) BD_VK(64, 4, 4, false, false)
+  BD_VK(128, 4, 1, false, false) BD_VK(128, 4, 2, false, false) BD_VK(128, 4, 4, false, false)
 #undef BD_VK
   return {nullptr, 0, 0};
 }
@@ -368,7 +461,7 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   const int nq_rows = group * n_q;
   const Variant v = pick_variant(nq_rows, with_v);
   if (v.nt == 0) return false;
-  const KernelInfo k = select_kernel(s.head_dim, v.nt, v.wq, with_v);
+  const KernelInfo k = select_kernel(s.head_dim, v.nt, v.wq, with_v, false);
   if (!k.fn) return false;
   plan->nq_rows = nq_rows;
   plan->nt = v.nt;
@@ -392,14 +485,6 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   if (vtotal >= (1L << 31)) return false;
   long vtpc = (vtotal + ctas - 1) / ctas;
   vtpc = std::max<long>(vtpc, (tpu + a + kVMaxSeg - 2) / (kVMaxSeg - 1));   // <= kVMaxSeg segments
-  // The unit's last CTA merges its segments in one round trip while they fit its staging
-  // area; beyond that the merge reads every part of every output element from L2 in turn,
-  // which costs far more than the streaming balance gains (a 4K context at batch 1: 16
-  // segments per unit, 24 us).  So, where the area holds two parts or more, a unit spans at
-  // most that many CTAs: a span of L tiles cut into ranges of v touches at most
-  // ceil((L - 1) / v) + 1 of them.
-  const long cap = with_v ? (long)(k.merge_floats / ((size_t)nq_rows * s.head_dim)) : 0;
-  if (cap >= 2) vtpc = std::max<long>(vtpc, (tpu + a - 1 + cap - 2) / (cap - 1));
   plan->seg_cost = a;
   plan->tiles_per_cta = (int)vtpc;
   plan->total_tiles = (int)total;
@@ -421,13 +506,17 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
     plan->smem_bytes += align_up((size_t)(units + 1) * 4, 16);
     if (plan->smem_bytes > 227 * 1024) return false;
   }
+  // the unit's last CTA merges its segments in one staged round trip while they fit its
+  // merge area; more segments take the chunked merge of the wide instance
+  plan->wide = with_v && (size_t)plan->max_seg * nq_rows * s.head_dim > k.merge_floats;
   return true;
 }
 
 size_t verify_partials_bytes(const bd_shape& s, const VerifyPlan& plan) {
   if (plan.max_seg <= 1) return 0;
   const size_t rows = (size_t)s.batch * s.h_kv * plan.max_seg * plan.nq_rows;
-  return align_up(rows * s.head_dim * 4, 256) + align_up(rows * 4, 256);
+  return align_up(rows * s.head_dim * 4, 256) + align_up(rows * 4, 256) +
+         (plan.wide ? align_up((size_t)s.batch * s.h_kv * 4, 256) : 0);
 }
 
 cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, const void* q,
@@ -451,6 +540,7 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.o_part = static_cast<float*>(ws_region);
   p.lse_part = reinterpret_cast<float*>(static_cast<uint8_t*>(ws_region) + align_up(rows * s.head_dim * 4, 256));
   p.counters = counters;
+  p.nseg = reinterpret_cast<int*>(reinterpret_cast<uint8_t*>(p.lse_part) + align_up(rows * 4, 256));
   p.status = status;
   p.n_q = n_q;
   p.nq_rows = plan.nq_rows;
@@ -464,11 +554,22 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.vtiles_per_cta = plan.tiles_per_cta;
   p.max_seg = plan.max_seg;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
-  const KernelInfo k = select_kernel(s.head_dim, plan.nt, plan.wq, plan.with_v);
+  const KernelInfo k = select_kernel(s.head_dim, plan.nt, plan.wq, plan.with_v, plan.wide);
   err = cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)plan.smem_bytes);
   if (err != cudaSuccess) return err;
   void* args[] = {&p, &kmap, &vmap};
-  return launch_kernel(k.fn, dim3(plan.grid), dim3(kVThreads), plan.smem_bytes, stream, args, 0);
+  err = launch_kernel(k.fn, dim3(plan.grid), dim3(kVThreads), plan.smem_bytes, stream, args, 0);
+  if (err != cudaSuccess || !plan.wide) return err;
+  const float* op = p.o_part;
+  const float* lp = p.lse_part;
+  const int* ns = p.nseg;
+  int max_seg = plan.max_seg, nq = plan.nq_rows;
+  __nv_bfloat16* o = p.o;
+  float* l = p.lse;
+  void* margs[] = {&op, &lp, &ns, &max_seg, &nq, &o, &l};
+  void* mfn = s.head_dim == 64 ? reinterpret_cast<void*>(&verify_merge_kernel<64>)
+                               : reinterpret_cast<void*>(&verify_merge_kernel<128>);
+  return launch_kernel(mfn, dim3(units, plan.nq_rows), dim3(128), 0, stream, margs, 0);
 }
 
 }  // namespace bd
