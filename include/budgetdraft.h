@@ -209,8 +209,9 @@ int bd_draft_attn_static(const bd_shape* shape, const void* q, const void* k_cac
  *   q        bf16 [batch, h_q, n_q, d]
  *   o_out    bf16 [batch, h_q, n_q, d], or NULL to compute lse only (V not read);
  *   lse_out  fp32 [batch, h_q, n_q] (may be NULL when o_out is not).
- * Constraints: 1 <= n_q, t_ctx + n_q <= t_cap, (h_q/h_kv)*n_q <= 96 (<= 128 when
- * o_out is NULL).
+ * Constraints: 1 <= n_q, t_ctx + n_q <= t_cap, (h_q/h_kv)*n_q <= 768 (<= 128 when
+ * o_out is NULL).  A KV head's query rows beyond 96 are processed in up to eight chunks
+ * of equal size that stream the same keys side by side.
  */
 int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_cache,
                    const void* v_cache, void* o_out, float* lse_out, void* ws, size_t ws_bytes,

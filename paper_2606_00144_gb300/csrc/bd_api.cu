@@ -259,8 +259,8 @@ int bd_verify_attn(const bd_shape* shape, const void* q, int n_q, const void* k_
   if (!o_out && !lse_out) return BD_ERR_INVALID_ARG;
   if (n_q < 1 || (long long)s.t_ctx + n_q > s.t_cap) return BD_ERR_INVALID_ARG;
   const bool with_v = o_out != nullptr;
-  const int nq_rows = (s.h_q / s.h_kv) * n_q;
-  if (nq_rows > (with_v ? 96 : 128)) return BD_ERR_UNSUPPORTED;
+  const long long nq_rows = (long long)(s.h_q / s.h_kv) * n_q;
+  if (nq_rows > (with_v ? 768 : 128)) return BD_ERR_UNSUPPORTED;
   VerifyPlan vp;
   if (!verify_plan(s, n_q, with_v, &vp)) return BD_ERR_UNSUPPORTED;
   if (!ws) return BD_ERR_WORKSPACE;

@@ -28,7 +28,9 @@ size_t ws_region_offset(int units);
 
 // ---------------------------------------------------------------------------- verify
 struct VerifyPlan {
-  int nq_rows;          // query rows per (sequence, KV head) = group * n_q
+  int nq_rows;          // query rows per unit (a chunk of the group * n_q rows of a KV head)
+  int rows_total;       // group * n_q
+  int row_chunks;       // chunks of a (sequence, KV head): units = batch * h_kv * row_chunks
   int nt, wq;           // n-tiles per warp, warp groups along queries
   int tiles_per_unit;   // 64-key tiles over [0, t_ctx + n_q)
   int total_tiles;      // over all units

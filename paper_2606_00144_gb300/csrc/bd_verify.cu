@@ -30,6 +30,8 @@ constexpr int kVConsumers = 4;        // consumer warps
 constexpr int kVThreads = 160;        // + one producer warp
 constexpr int kVStages = 5;
 constexpr int kVMaxSeg = 33;          // bound on the segments of one unit
+constexpr int kVMaxRows = 96;         // query rows one CTA's consumer warps hold (with V)
+constexpr int kVMaxChunks = 8;        // row chunks of one (sequence, KV head)
 
 struct VerifyParams {
   const __nv_bfloat16* q;
@@ -44,6 +46,12 @@ struct VerifyParams {
   int h_kv;
   int len_offset;      // added to every length (the window LSE pass runs at T - W)
   int n_q, nq_rows, t_ctx, tiles_per_unit, total_tiles, max_seg;
+  // Query rows of a (sequence, KV head) beyond what one CTA's warps hold are cut into
+  // row_chunks chunks of nq_rows rows (the last may hold fewer): a "unit" below is one
+  // (sequence, KV head, chunk), and a KV head's chunks are adjacent in the unit list, so
+  // CTAs streaming the same keys run side by side (the second read hits L2).
+  int rows_total;      // group * n_q
+  int row_chunks;
   int seg_cost;        // virtual tiles charged for each unit a CTA starts (see verify_plan)
   int vtiles_per_cta;  // contiguous range of the virtual tile list per CTA
   float scale_log2;    // log2(e) / sqrt(D)
@@ -136,7 +144,8 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     const int per = (n_units + kVThreads - 1) / kVThreads;
     const int u0 = min(n_units, tid * per), u1 = min(n_units, u0 + per);
     auto span = [&](int u) {
-      const int t_u = max(0, unit_context(p.seq_lens, u, p.h_kv, p.t_ctx - p.len_offset, nullptr) + p.len_offset);
+      const int t_u =
+          max(0, unit_context(p.seq_lens, u / p.row_chunks, p.h_kv, p.t_ctx - p.len_offset, nullptr) + p.len_offset);
       return (t_u + p.n_q + kVKeys - 1) / kVKeys + p.seg_cost;
     };
     int sum = 0;
@@ -187,6 +196,7 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
       bool stop = false;
       for (int unit = u_first; unit <= u_last && !stop; ++unit) {
         const int tb = map.first_tile(unit, v0), te = map.end_tile(unit, v1);
+        const int kv_unit = unit / p.row_chunks;
         for (int tile = tb; tile < te; ++tile) {
           const int t = issued;
           const int s = t % STAGES;
@@ -202,11 +212,11 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
           uint8_t* st = stage_base + s * L::STAGE_BYTES;
           mbar_arrive_expect_tx(&full_bar[s], L::STAGE_BYTES);
 #pragma unroll
-          for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * HALF_BYTES, &kmap, &full_bar[s], 64 * h, key0, unit);
+          for (int h = 0; h < D / 64; ++h) tma_load_3d(st + h * HALF_BYTES, &kmap, &full_bar[s], 64 * h, key0, kv_unit);
           if (WITH_V) {
 #pragma unroll
             for (int h = 0; h < D / 64; ++h)
-              tma_load_3d(st + L::TILE_BYTES + h * HALF_BYTES, &vmap, &full_bar[s], 64 * h, key0, unit);
+              tma_load_3d(st + L::TILE_BYTES + h * HALF_BYTES, &vmap, &full_bar[s], 64 * h, key0, kv_unit);
           }
           issued = t + 1;
         }
@@ -221,12 +231,13 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
 
   // -------------------------------------------------------------------- consumers
   if (!p.seq_lens)   // the first unit's queries on their way into L2 while the predecessor finishes
-    prefetch_lines_l2(p.q + (size_t)u_first * p.nq_rows * D, (size_t)p.nq_rows * D * 2, tid, kVConsumers * 32);
+    prefetch_lines_l2(p.q + ((size_t)(u_first / p.row_chunks) * p.rows_total + (u_first % p.row_chunks) * p.nq_rows) * D,
+                      (size_t)p.nq_rows * D * 2, tid, kVConsumers * 32);
   grid_dependency_wait();                        // the queries come from the preceding kernels
   allow_dependent_launch();
   const int wq = warp % WQ, wk = warp / WQ;
   const int tig = lane & 3;
-  const int nq = p.nq_rows;
+  const int nq = p.nq_rows;                      // rows per unit slot (the chunk size)
   constexpr int NCT = kVConsumers * 32;          // consumer threads
   int lim[NT][2];                                // last visible key of each of this thread's columns
 
@@ -235,17 +246,21 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
   for (int unit = u_first; unit <= u_last; ++unit) {
     const int tb = map.first_tile(unit, v0), te = map.end_tile(unit, v1);
     if (tb >= te) continue;                      // only virtual tiles of this unit here
-    const int t_unit = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx - p.len_offset, tid == 0 ? p.status : nullptr) +
-                       p.len_offset;
+    const int kv_unit = unit / p.row_chunks;
+    const int row_base = (unit - kv_unit * p.row_chunks) * nq;   // first row of this chunk
+    const int rows = min(nq, p.rows_total - row_base);
+    const size_t row0 = (size_t)kv_unit * p.rows_total + row_base;   // its first row in q / o / lse
+    const int t_unit =
+        unit_context(p.seq_lens, kv_unit, p.h_kv, p.t_ctx - p.len_offset, tid == 0 ? p.status : nullptr) + p.len_offset;
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
         const int col = 8 * (wq * NT + nt) + 2 * tig + e;
-        lim[nt][e] = col < nq ? t_unit + col % p.n_q : -1;
+        lim[nt][e] = col < rows ? t_unit + (row_base + col) % p.n_q : -1;
       }
     uint32_t bq[NT][D / 16][2];
-    WarpAttn<D, NT, WITH_V>::load_q(bq, p.q + (size_t)unit * nq * D, nq, wq * NT, lane);
+    WarpAttn<D, NT, WITH_V>::load_q(bq, p.q + row0 * D, rows, wq * NT, lane);
     WarpAttn<D, NT, WITH_V> wa;
     wa.init();
     for (int tile = tb; tile < te && alive; ++tile, ++t) {
@@ -276,19 +291,18 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     const int c_first = map.owner(unit, 0);
     const int c_last = map.owner(unit, map.tiles(unit) - 1);
     const int n_seg = c_last - c_first + 1;
-    const size_t row0 = (size_t)unit * nq;
     if (WIDE && c == c_first && tid == 0) p.nseg[unit] = n_seg;
     if (n_seg == 1) {
-      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, nq, p.lse ? p.lse + row0 : nullptr,
+      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, rows, p.lse ? p.lse + row0 : nullptr,
                                            WITH_V ? static_cast<void*>(p.o + row0 * D) : nullptr, true, tid, NCT, 1);
     } else if constexpr (WIDE) {
       const size_t slot = (size_t)unit * p.max_seg + (c - c_first);
-      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, nq, p.lse_part + slot * nq,
+      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, rows, p.lse_part + slot * nq,
                                            WITH_V ? static_cast<void*>(p.o_part + slot * nq * D) : nullptr, false,
                                            tid, NCT, 1);
     } else {
       const size_t slot = (size_t)unit * p.max_seg + (c - c_first);
-      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, nq, p.lse_part + slot * nq,
+      merge_warps_and_store<D, WK, WITH_V>(m_s, l_s, f_s, o_s, NQC, rows, p.lse_part + slot * nq,
                                            WITH_V ? static_cast<void*>(p.o_part + slot * nq * D) : nullptr, false,
                                            tid, NCT, 1);
       __threadfence();
@@ -298,7 +312,7 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
       if (*last_flag) {
         __threadfence();
         const size_t base = (size_t)unit * p.max_seg;
-        merge_partials<D>(p.o_part + base * nq * D, p.lse_part + base * nq, n_seg, nq, (size_t)nq * D, (size_t)nq,
+        merge_partials<D>(p.o_part + base * nq * D, p.lse_part + base * nq, n_seg, rows, (size_t)nq * D, (size_t)nq,
                           WITH_V ? p.o + row0 * D : nullptr, p.lse ? p.lse + row0 : nullptr, [](int r) { return r; },
                           w_s, tid, NCT, 1, m_s, L::kMerge / 4);
         if (tid == 0) p.counters[unit] = 0;
@@ -319,8 +333,8 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
 // trips to L2 in all; the groups' sums meet in shared memory.
 template <int D>
 __global__ void __launch_bounds__(128) verify_merge_kernel(const float* o_part, const float* lse_part,
-                                                           const int* nseg, int max_seg, int nq,
-                                                           __nv_bfloat16* o, float* lse) {
+                                                           const int* nseg, int max_seg, int nq, int rows_total,
+                                                           int row_chunks, __nv_bfloat16* o, float* lse) {
   constexpr int Q = D / 4;                 // column quads per row
   constexpr int NG = 128 / Q;              // segment groups
   constexpr int PER = (kVMaxSeg + NG - 1) / NG;
@@ -329,8 +343,10 @@ __global__ void __launch_bounds__(128) verify_merge_kernel(const float* o_part, 
   __shared__ float w[kVMaxSeg];
   __shared__ float4 part[NG][Q];
   const int unit = blockIdx.x, r = blockIdx.y, tid = threadIdx.x;
+  const int kv_unit = unit / row_chunks, row_base = (unit - kv_unit * row_chunks) * nq;
   const int n = min(__ldcg(nseg + unit), kVMaxSeg);
-  if (n <= 1) return;
+  if (n <= 1 || row_base + r >= rows_total) return;
+  const size_t orow = (size_t)kv_unit * rows_total + row_base + r;   // the output row
   const size_t base = (size_t)unit * max_seg;
   if (tid < 32) {
     const float l0 = tid < n ? __ldcg(lse_part + (base + tid) * nq + r) : -INFINITY;
@@ -346,7 +362,7 @@ __global__ void __launch_bounds__(128) verify_merge_kernel(const float* o_part, 
     const float inv = tot > 0.f ? 1.f / tot : 0.f;
     if (tid < n) w[tid] = e0 * inv;
     if (tid + 32 < n) w[tid + 32] = e1 * inv;
-    if (tid == 0 && lse) lse[(size_t)unit * nq + r] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
+    if (tid == 0 && lse) lse[orow] = mx == -INFINITY ? -INFINITY : mx + logf(tot);
   }
   if (o == nullptr) return;
   const int q = tid % Q, g = tid / Q;
@@ -384,7 +400,7 @@ __global__ void __launch_bounds__(128) verify_merge_kernel(const float* o_part, 
     uint2 packed;
     packed.x = pack_bf16x2(acc.x, acc.y);
     packed.y = pack_bf16x2(acc.z, acc.w);
-    *reinterpret_cast<uint2*>(o + ((size_t)unit * nq + r) * D + 4 * q) = packed;
+    *reinterpret_cast<uint2*>(o + orow * D + 4 * q) = packed;
   }
 }
 
@@ -458,12 +474,18 @@ int occupancy(const KernelInfo& k) {
 
 bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   const int group = s.h_q / s.h_kv;
-  const int nq_rows = group * n_q;
+  const long rows_total = (long)group * n_q;
+  // more query rows than one CTA's warps hold (96 with V): chunks of equal size
+  const int chunks = with_v && rows_total > kVMaxRows ? (int)((rows_total + kVMaxRows - 1) / kVMaxRows) : 1;
+  if (chunks > kVMaxChunks) return false;
+  const int nq_rows = (int)((rows_total + chunks - 1) / chunks);
   const Variant v = pick_variant(nq_rows, with_v);
   if (v.nt == 0) return false;
   const KernelInfo k = select_kernel(s.head_dim, v.nt, v.wq, with_v, false);
   if (!k.fn) return false;
   plan->nq_rows = nq_rows;
+  plan->rows_total = (int)rows_total;
+  plan->row_chunks = chunks;
   plan->nt = v.nt;
   plan->wq = v.wq;
   plan->with_v = with_v;
@@ -471,7 +493,7 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   plan->smem_bytes = k.smem;
   const long n_keys = (long)s.t_ctx + n_q;
   plan->tiles_per_unit = (int)((n_keys + kVKeys - 1) / kVKeys);
-  const long units = (long)s.batch * s.h_kv;
+  const long units = (long)s.batch * s.h_kv * chunks;
   const int tpu = plan->tiles_per_unit;
   const long total = units * tpu;
   const long ctas = std::max(1, current_sm_count() * occupancy(k));
@@ -508,15 +530,16 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   }
   // the unit's last CTA merges its segments in one staged round trip while they fit its
   // merge area; more segments take the chunked merge of the wide instance
-  plan->wide = with_v && (size_t)plan->max_seg * nq_rows * s.head_dim > k.merge_floats;
+  plan->wide = with_v && ((size_t)plan->max_seg * nq_rows * s.head_dim > k.merge_floats ||
+                          (chunks > 1 && plan->max_seg > 1));   // the chunks' units have no arrival counters
   return true;
 }
 
 size_t verify_partials_bytes(const bd_shape& s, const VerifyPlan& plan) {
   if (plan.max_seg <= 1) return 0;
-  const size_t rows = (size_t)s.batch * s.h_kv * plan.max_seg * plan.nq_rows;
-  return align_up(rows * s.head_dim * 4, 256) + align_up(rows * 4, 256) +
-         (plan.wide ? align_up((size_t)s.batch * s.h_kv * 4, 256) : 0);
+  const size_t units = (size_t)s.batch * s.h_kv * plan.row_chunks;
+  const size_t rows = units * plan.max_seg * plan.nq_rows;
+  return align_up(rows * s.head_dim * 4, 256) + align_up(rows * 4, 256) + (plan.wide ? align_up(units * 4, 256) : 0);
 }
 
 cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, const void* q,
@@ -536,7 +559,7 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.q = static_cast<const __nv_bfloat16*>(q);
   p.o = static_cast<__nv_bfloat16*>(o_out);
   p.lse = lse_out;
-  const size_t rows = (size_t)units * plan.max_seg * plan.nq_rows;
+  const size_t rows = (size_t)units * plan.row_chunks * plan.max_seg * plan.nq_rows;
   p.o_part = static_cast<float*>(ws_region);
   p.lse_part = reinterpret_cast<float*>(static_cast<uint8_t*>(ws_region) + align_up(rows * s.head_dim * 4, 256));
   p.counters = counters;
@@ -544,6 +567,8 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   p.status = status;
   p.n_q = n_q;
   p.nq_rows = plan.nq_rows;
+  p.rows_total = plan.rows_total;
+  p.row_chunks = plan.row_chunks;
   p.t_ctx = s.t_ctx;
   p.seq_lens = s.seq_lens;
   p.h_kv = s.h_kv;
@@ -563,13 +588,13 @@ cudaError_t launch_verify(const bd_shape& s, const VerifyPlan& plan, int n_q, co
   const float* op = p.o_part;
   const float* lp = p.lse_part;
   const int* ns = p.nseg;
-  int max_seg = plan.max_seg, nq = plan.nq_rows;
+  int max_seg = plan.max_seg, nq = plan.nq_rows, rows_total = plan.rows_total, chunks = plan.row_chunks;
   __nv_bfloat16* o = p.o;
   float* l = p.lse;
-  void* margs[] = {&op, &lp, &ns, &max_seg, &nq, &o, &l};
+  void* margs[] = {&op, &lp, &ns, &max_seg, &nq, &rows_total, &chunks, &o, &l};
   void* mfn = s.head_dim == 64 ? reinterpret_cast<void*>(&verify_merge_kernel<64>)
                                : reinterpret_cast<void*>(&verify_merge_kernel<128>);
-  return launch_kernel(mfn, dim3(units, plan.nq_rows), dim3(128), 0, stream, margs, 0);
+  return launch_kernel(mfn, dim3(units * plan.row_chunks, plan.nq_rows), dim3(128), 0, stream, margs, 0);
 }
 
 }  // namespace bd

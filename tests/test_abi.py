@@ -78,7 +78,7 @@ def test_verify_validation(lib):
     assert verify(lib, shape(), n_q=0) == INVALID
     assert verify(lib, shape(), n_q=11) == INVALID                    # t_ctx + n_q > t_cap
     assert verify(lib, shape(), o=0, lse=0) == INVALID                # nothing to write
-    assert verify(lib, shape(t_cap=200), n_q=25) == UNSUPPORTED       # 4 * 25 rows > 96 with V
+    assert verify(lib, shape(t_cap=400), n_q=193) == UNSUPPORTED      # 4 * 193 rows > 768 with V
     assert verify(lib, shape(t_cap=200), n_q=33, o=0) == UNSUPPORTED  # 4 * 33 rows > 128, lse only
 
 

@@ -220,7 +220,8 @@ def test_ragged_shapes(case):
 def test_verify_block_sizes(n_q, with_v):
     wl = W.tiny_workload(batch=2, h_q=8, h_kv=2, head_dim=128, t_ctx=1500, gamma=n_q - 1 if n_q > 1 else 1)
     inp = W.make_layer(wl, 0, "cuda")
-    q = torch.randn(wl.batch, wl.h_q, n_q, wl.head_dim, device="cuda").to(torch.bfloat16)
+    g = torch.Generator(device="cuda").manual_seed(900 + n_q)
+    q = torch.randn(wl.batch, wl.h_q, n_q, wl.head_dim, device="cuda", generator=g).to(torch.bfloat16)
     shape = bd.shape_of(inp.k_cache, wl.h_q, wl.t_ctx)
     ws = bd.Workspace(bd.bd_workspace_size(shape, bd.BD_OP_VERIFY, 1, n_q))
     o = torch.empty(wl.batch, wl.h_q, n_q, wl.head_dim, dtype=torch.bfloat16, device="cuda") if with_v else None
@@ -232,6 +233,50 @@ def test_verify_block_sizes(n_q, with_v):
         check_attention(o, lse, o_ref, l_ref, f"verify n_q={n_q}")
     else:
         assert np.abs(f64(lse) - l_ref).max() <= 1e-3
+
+
+@pytest.mark.parametrize("h_q,h_kv,d,t_ctx,n_q", [(32, 4, 128, 1500, 21), (32, 4, 64, 777, 13), (32, 2, 128, 900, 21),
+                                                   (32, 4, 128, 16384, 21)])
+def test_verify_blocks_beyond_one_cta(h_q, h_kv, d, t_ctx, n_q):
+    """More query rows per KV head than one CTA's warps hold (96): G = 8 with the paper's
+    gamma = 20 (168 rows, two chunks), 104 rows, and G = 16 (336 rows, four chunks), the last
+    case at 16K context."""
+    wl = W.tiny_workload(batch=2, h_q=h_q, h_kv=h_kv, head_dim=d, t_ctx=t_ctx, gamma=n_q - 1)
+    inp = W.make_layer(wl, 0, "cuda")
+    g = torch.Generator(device="cuda").manual_seed(4242 + n_q)
+    q = torch.randn(wl.batch, wl.h_q, n_q, d, device="cuda", generator=g).to(torch.bfloat16)
+    shape = bd.shape_of(inp.k_cache, wl.h_q, wl.t_ctx)
+    ws = bd.Workspace(bd.bd_workspace_size(shape, bd.BD_OP_VERIFY, 1, n_q))
+    o = torch.empty(wl.batch, wl.h_q, n_q, d, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(wl.batch, wl.h_q, n_q, device="cuda")
+    for rep in range(2):                       # the workspace is reused as in a loop of steps
+        o.fill_(7)
+        bd.bd_verify_attn(shape, q, n_q, inp.k_cache, inp.v_cache, o, lse, ws)
+        torch.cuda.synchronize()
+        o_ref, l_ref = oracle.verify_attn(f64(q), f64(inp.k_cache), f64(inp.v_cache), wl.t_ctx)
+        check_attention(o, lse, o_ref, l_ref, f"verify G={h_q // h_kv} n_q={n_q} T={t_ctx} rep {rep}")
+    assert ws.status() == 0
+
+
+def test_verify_chunked_block_with_per_sequence_lengths():
+    lens = [1500, 977, 64]
+    b, h_q, h_kv, d, n_q = len(lens), 32, 4, 128, 21
+    wl = W.tiny_workload(batch=b, h_q=h_q, h_kv=h_kv, head_dim=d, t_ctx=max(lens), gamma=n_q - 1)
+    inp = W.make_layer(wl, 0, "cuda")
+    g = torch.Generator(device="cuda").manual_seed(77)
+    q = torch.randn(b, h_q, n_q, d, device="cuda", generator=g).to(torch.bfloat16)
+    lens_d = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    shape = bd.make_shape(b, h_q, h_kv, d, max(lens), wl.t_cap, seq_lens=lens_d)
+    ws = bd.Workspace(bd.bd_workspace_size(shape, bd.BD_OP_VERIFY, 1, n_q))
+    o = torch.empty(b, h_q, n_q, d, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(b, h_q, n_q, device="cuda")
+    bd.bd_verify_attn(shape, q, n_q, inp.k_cache, inp.v_cache, o, lse, ws)
+    torch.cuda.synchronize()
+    K, V, Q = f64(inp.k_cache), f64(inp.v_cache), f64(q)
+    for i, t in enumerate(lens):
+        o_ref, l_ref = oracle.verify_attn(Q[i:i + 1], K[i:i + 1], V[i:i + 1], t)
+        check_attention(o[i:i + 1], lse[i:i + 1], o_ref, l_ref, f"chunked verify seq {i} T={t}")
+    assert ws.status() == 0
 
 
 def test_draft_empty_view_and_full_view():
