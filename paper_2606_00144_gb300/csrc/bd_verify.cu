@@ -243,9 +243,22 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
 
   bool alive = true;   // false once this warp's wait gave up (the abort flag is then set)
   int t = 0;
-  for (int unit = u_first; unit <= u_last; ++unit) {
+  // the next unit of this range with real tiles here (past u_last: none)
+  auto next_unit = [&](int u) {
+    while (u <= u_last && map.first_tile(u, v0) >= map.end_tile(u, v1)) ++u;
+    return u;
+  };
+  // the unit's queries: a chunk of rows of its KV head's block
+  auto unit_q = [&](int u, uint32_t (&bq)[NT][D / 16][2]) {
+    const int kv = u / p.row_chunks, base = (u - kv * p.row_chunks) * nq;
+    WarpAttn<D, NT, WITH_V>::load_q(bq, p.q + ((size_t)kv * p.rows_total + base) * D, min(nq, p.rows_total - base),
+                                    wq * NT, lane);
+  };
+  uint32_t bq[NT][D / 16][2];
+  int unit = next_unit(u_first);
+  if (unit <= u_last) unit_q(unit, bq);
+  for (; unit <= u_last;) {
     const int tb = map.first_tile(unit, v0), te = map.end_tile(unit, v1);
-    if (tb >= te) continue;                      // only virtual tiles of this unit here
     const int kv_unit = unit / p.row_chunks;
     const int row_base = (unit - kv_unit * p.row_chunks) * nq;   // first row of this chunk
     const int rows = min(nq, p.rows_total - row_base);
@@ -259,8 +272,6 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
         const int col = 8 * (wq * NT + nt) + 2 * tig + e;
         lim[nt][e] = col < rows ? t_unit + (row_base + col) % p.n_q : -1;
       }
-    uint32_t bq[NT][D / 16][2];
-    WarpAttn<D, NT, WITH_V>::load_q(bq, p.q + row0 * D, rows, wq * NT, lane);
     WarpAttn<D, NT, WITH_V> wa;
     wa.init();
     for (int tile = tb; tile < te && alive; ++tile, ++t) {
@@ -282,6 +293,10 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
       __syncwarp();
       if (lane == 0) mbar_arrive(&empty_bar[s]);
     }
+    // the next unit's queries are requested now, so that they arrive while this segment
+    // closes (its merge, partial write and arrival take several round trips to memory)
+    const int next = next_unit(unit + 1);
+    if (next <= u_last && alive) unit_q(next, bq);
     wa.finish_rows();
 
     // ---------------------------------------------------------------- end of a segment
@@ -323,6 +338,7 @@ __global__ void __launch_bounds__(kVThreads) verify_kernel(const VerifyParams p,
     if (tid == 0) last_flag[1] = *abort_flag;
     named_bar(1, NCT);
     if (last_flag[1]) break;
+    unit = next;
   }
 }
 
@@ -497,12 +513,14 @@ bool verify_plan(const bd_shape& s, int n_q, bool with_v, VerifyPlan* plan) {
   const int tpu = plan->tiles_per_unit;
   const long total = units * tpu;
   const long ctas = std::max(1, current_sm_count() * occupancy(k));
-  // A segment end (merge of the warps' partials, its write, the arrival, the next unit's
-  // queries) costs about 3 us of streaming time; charge it as virtual tiles at the rate
-  // one CTA streams at when every SM streams (measured ~6.5 TB/s over all SMs).
+  // A unit boundary inside a CTA's range (the segment's merge of the warps' partials, its
+  // write, the arrival, the merge by the unit's last CTA) costs about 5 us of streaming time;
+  // charge it as virtual tiles at the rate one CTA streams at when every SM streams
+  // (~6.5 TB/s over all SMs).  Traced: with 3 us charged, the CTAs holding a boundary ended
+  // their last tile ~5 us after the others; swept at 1-12 us, 5 us gave the shortest step.
   const double tile_bytes = (double)kVKeys * s.head_dim * 2 * (with_v ? 2 : 1);
   const double tile_us = tile_bytes / (6.5e6 / (double)std::max(1, current_sm_count()));
-  const int a = (int)std::min(16.0, std::max(0.0, 3.0 / tile_us + 0.5));
+  const int a = (int)std::min(16.0, std::max(0.0, 5.0 / tile_us + 0.5));
   const long vtotal = units * (tpu + a);
   if (vtotal >= (1L << 31)) return false;
   long vtpc = (vtotal + ctas - 1) / ctas;
