@@ -21,7 +21,8 @@
  *   bd_advance        slides the observation window over the settled block rows and
  *                     appends their positions to the sparse view (Algorithm 2, Update).
  * Around them: bd_workspace_size / bd_workspace_status (scratch and device-side
- * errors), bd_draft_attn_static (bd_draft_attn without a workspace),
+ * errors), bd_draft_attn_static / bd_draft_static_status (bd_draft_attn without a
+ * workspace, and its error word),
  * bd_check_wait_timeout (runs the device-side error path on purpose) and bd_strerror.
  *
  * Conventions shared by every call
@@ -192,9 +193,9 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
  *     current (cudaGetSymbolAddress); make that first call before any stream capture.
  *     The address is kept for the life of the process: after cudaDeviceReset on a device
  *     this entry point has been called on, it must not be called on that device again.
- *   - Every call clears the array's status word and counters on `stream` before its
- *     kernel.  Out-of-range indices are skipped as in bd_draft_attn, but this variant
- *     does not report device-side errors.
+ *   - Every call clears the array's counters on `stream` before its kernel.  Device-side
+ *     errors (an index outside the context, which is skipped as in bd_draft_attn) set the
+ *     array's status word, which keeps them until bd_draft_static_status reads it.
  *   - All calls share the one array: calls whose work can overlap on the GPU (different
  *     streams, or threads without ordering between them) race and corrupt each other's
  *     results.  Issue them on one stream.
@@ -202,6 +203,14 @@ int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, con
 int bd_draft_attn_static(const bd_shape* shape, const void* q, const void* k_cache,
                          const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
                          int step_j, void* o_out, float* lse_out, void* stream);
+
+/*
+ * Status word of bd_draft_attn_static's array on the current device (no counterpart in
+ * the paper): waits for `stream`, returns the first device-side error the calls on it
+ * recorded since the last read (BD_OK if none) and clears it.  Call it on the stream
+ * the static calls were issued on.
+ */
+int bd_draft_static_status(void* stream);
 
 /*
  * Verifier block attention (Algorithm 2, Verify): query i (0 <= i < n_q) of head h

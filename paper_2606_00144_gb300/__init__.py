@@ -25,6 +25,7 @@ from .binding import (  # noqa: F401
     bd_combine,
     bd_draft_attn,
     bd_draft_attn_static,
+    bd_draft_static_status,
     bd_select_budget,
     bd_strerror,
     bd_verify_attn,

@@ -15,6 +15,7 @@ import torch
 from .build import LIB_PATH
 
 BD_OK = 0
+BD_ERR_CUDA = -5
 BD_OP_SELECT, BD_OP_DRAFT, BD_OP_VERIFY = 1, 2, 3
 BD_DRAFT_VIEW_READY = 1
 BD_SELECT_WINDOW_READY = 1
@@ -49,6 +50,7 @@ _SIGNATURES = {
                                      _P, _P, ctypes.c_size_t, _P]),
     "bd_draft_attn_static": (ctypes.c_int, [_SHAPE, _P, _P, _P, _P, _P, ctypes.c_int, ctypes.c_int, _P, _P,
                                             _P]),
+    "bd_draft_static_status": (ctypes.c_int, [_P]),
     "bd_verify_attn": (ctypes.c_int, [_SHAPE, _P, ctypes.c_int, _P, _P, _P, _P, _P, ctypes.c_size_t, _P]),
     "bd_combine": (ctypes.c_int, [_P, _P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P, _P]),
     "bd_argmax": (ctypes.c_int, [_P, ctypes.c_int, ctypes.c_int, ctypes.c_int, _P, _P]),
@@ -171,6 +173,14 @@ def bd_draft_attn_static(shape, q, k_cache, v_cache, idx, count, budget, step_j,
                                         _ptr(count), int(budget), int(step_j), _ptr(o_out), _ptr(lse_out),
                                         _stream(stream))
     _check("bd_draft_attn_static", st)
+
+
+def bd_draft_static_status(stream=None) -> int:
+    """Reads and clears the device-side error word of bd_draft_attn_static's array."""
+    st = library().bd_draft_static_status(_stream(stream))
+    if st == BD_ERR_CUDA:
+        _check("bd_draft_static_status", st)
+    return int(st)
 
 
 def bd_verify_attn(shape, q, n_q, k_cache, v_cache, o_out, lse_out, ws: Workspace, stream=None):

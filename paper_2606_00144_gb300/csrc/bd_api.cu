@@ -370,6 +370,12 @@ int bd_check_wait_timeout(void* ws, size_t ws_bytes, int limit_us, void* stream)
   return map_cuda(launch_wait_probe(status_word(ws), limit_us, static_cast<cudaStream_t>(stream)));
 }
 
+int bd_draft_static_status(void* stream) {
+  int host = 0;
+  if (draft_static_status(&host, static_cast<cudaStream_t>(stream)) != cudaSuccess) return BD_ERR_CUDA;
+  return host;
+}
+
 int bd_workspace_status(void* ws, void* stream) {
   if (!ws) return BD_ERR_INVALID_ARG;
   int host = 0;

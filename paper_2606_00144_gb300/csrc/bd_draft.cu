@@ -390,13 +390,30 @@ cudaError_t launch_draft_static(const bd_shape& s, const DraftPlan& plan, const 
   if (err != cudaSuccess) return err;
   const int units = s.batch * s.h_kv;
   uint8_t* b = static_cast<uint8_t*>(base);
-  // The array keeps whatever the previous call left: clear the status word and the
-  // arrival counters (they must start at zero) before this call's kernel.
-  err = cudaMemsetAsync(b, 0, ws_region_offset(units), stream);
+  // The array keeps whatever the previous call left: clear the arrival counters (they
+  // must start at zero) before this call's kernel.  The status word keeps the errors of
+  // earlier calls until draft_static_status reads it.
+  err = cudaMemsetAsync(b + ws_counters_offset(), 0, ws_region_offset(units) - ws_counters_offset(), stream);
   if (err != cudaSuccess) return err;
   return launch_draft(s, plan, q, k_cache, v_cache, idx, count, budget, step_j, 0u, o_out, lse_out,
                       b + ws_region_offset(units), reinterpret_cast<int*>(b + ws_counters_offset()),
                       reinterpret_cast<int*>(b), stream);
+}
+
+// Reads and clears the array's status word on `stream` (after the calls queued on it).
+cudaError_t draft_static_status(int* out, cudaStream_t stream) {
+  void* base = nullptr;
+  cudaError_t err = draft_scratch_address(&base);
+  if (err != cudaSuccess) return err;
+  int host = 0;
+  err = cudaMemcpyAsync(&host, base, sizeof(int), cudaMemcpyDeviceToHost, stream);
+  if (err != cudaSuccess) return err;
+  err = cudaMemsetAsync(base, 0, sizeof(int), stream);
+  if (err != cudaSuccess) return err;
+  err = cudaStreamSynchronize(stream);
+  if (err != cudaSuccess) return err;
+  *out = host;
+  return cudaSuccess;
 }
 
 }  // namespace bd

@@ -65,6 +65,7 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
 
 // Allocation-free variant: scratch in a file-scope device array of this many bytes.
 size_t draft_static_scratch_bytes();
+cudaError_t draft_static_status(int* out, cudaStream_t stream);
 cudaError_t launch_draft_static(const bd_shape& s, const DraftPlan& plan, const void* q, const void* k_cache,
                                 const void* v_cache, const int32_t* idx, const int32_t* count, int budget,
                                 int step_j, void* o_out, float* lse_out, cudaStream_t stream);

@@ -55,6 +55,29 @@ def test_draft_attn_static_matches_oracle(budget):
     assert st.ws.status() == 0
 
 
+def test_draft_attn_static_reports_device_errors_until_read():
+    """The array's status word keeps a device-side error of a static call (an index past the
+    context, skipped like in bd_draft_attn) until bd_draft_static_status reads and clears it;
+    clean calls leave it at zero."""
+    bd.build()
+    wl = W.tiny_workload(batch=1, h_q=4, h_kv=1, head_dim=64, t_ctx=100, budget=8)
+    inp = W.make_layer(wl, 0, "cuda")
+    st = bd.SpecStep.for_workload(wl)
+    o = torch.empty(1, 4, 64, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(1, 4, device="cuda")
+    st.count.fill_(4)
+    assert bd.bd_draft_static_status() in (0, -1)          # whatever earlier calls left, now cleared
+    st.idx.copy_(torch.tensor([[[0, 5, 9, 20, -1, -1, -1, -1]]], dtype=torch.int32))
+    bd.bd_draft_attn_static(st.shape, inp.q_draft[0], inp.k_cache, inp.v_cache, st.idx, st.count, 8, 0, o, lse)
+    assert bd.bd_draft_static_status() == 0
+    st.idx.copy_(torch.tensor([[[0, 5, 100000, 20, -1, -1, -1, -1]]], dtype=torch.int32))
+    bd.bd_draft_attn_static(st.shape, inp.q_draft[0], inp.k_cache, inp.v_cache, st.idx, st.count, 8, 0, o, lse)
+    st.idx.copy_(torch.tensor([[[0, 5, 9, 20, -1, -1, -1, -1]]], dtype=torch.int32))
+    bd.bd_draft_attn_static(st.shape, inp.q_draft[0], inp.k_cache, inp.v_cache, st.idx, st.count, 8, 0, o, lse)
+    assert bd.bd_draft_static_status() == -1                # BD_ERR_INVALID_ARG, kept across the clean call
+    assert bd.bd_draft_static_status() == 0                 # reading clears it
+
+
 def test_draft_attn_static_rejects_oversized_scratch():
     bd.build()
     # 4 MiB is enough for the counters of ~1M (sequence, KV head) units but not 2M
