@@ -772,7 +772,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_kernel(const TopkParams 
   extern __shared__ uint32_t vals[];           // item values (fp32 bits) | candidates | samples
   __shared__ uint32_t hist[256];
   __shared__ uint32_t wsum[32];
-  __shared__ uint32_t s_total, s_prefix, s_krem, s_cnt;
+  __shared__ uint32_t s_total, s_prefix, s_krem;
   grid_dependency_wait();
   allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
