@@ -65,6 +65,13 @@ def step_bytes(wl, budget, n_recent, sel_mode, n_sink=None):
     return dict(select=sel, draft=draft, verify=verify, total=sel + draft + verify)
 
 
+def view_rereads(wl):
+    """Bytes of a step's sparse views read again by draft passes 2..gamma over all layers:
+    counted for a stack, whose per-pass views together are far above L2."""
+    view = min(wl.budget, wl.t_ctx) * 2 * wl.head_dim * 2 * wl.batch * wl.h_kv * wl.layers
+    return (wl.gamma - 1) * view
+
+
 # ----------------------------------------------------------------------------- clocks
 
 class ClockSampler:
@@ -552,11 +559,9 @@ def config_table(head, args, head_us, peak):
                       "bytes_per_step": b, "GB/s": round(gbs, 1), "pct_of_8tbs": round(100 * gbs / NOMINAL_HBM_GBS, 1),
                       "frac_of_measured_hbm": round(gbs / peak, 3)}
         if wl.layers > 1:
-            # a stack's per-pass sparse views (one layer's alone is far above L2) are read
-            # again by each of the gamma passes: the bytes with the view counted gamma times
-            units = wl.batch * wl.h_kv
-            view = min(wl.budget, wl.t_ctx) * 2 * wl.head_dim * 2 * units * wl.layers
-            bg = b + (wl.gamma - 1) * view
+            # a stack's per-pass sparse views are read again by each of the gamma passes:
+            # the bytes with the views counted gamma times
+            bg = b + view_rereads(wl)
             gbg = bg / (us * 1e-6) / 1e9
             rows[name].update({"bytes_per_step_views_x_gamma": bg, "GB/s_views_x_gamma": round(gbg, 1),
                                "frac_of_measured_hbm_views_x_gamma": round(gbg / peak, 3)})
