@@ -401,6 +401,42 @@ def test_boundary_among_underflowed_scores():
     run_and_check(wl, inp, host(inp), check_steps=False, tag="boundary among zero scores")
 
 
+@pytest.mark.parametrize("run", [4, 64])
+def test_exact_ties_ranked_above_the_bound(run):
+    """Middle keys repeated in runs of `run` identical rows, so scores tie exactly in runs,
+    and the top-B that ranks only the scores above the bound from group maxima meets its
+    boundary inside a run (k = 266 is no multiple of 4): four ties in the boundary bin
+    (ranked by one warp) or 64 (ranked by the whole CTA).  Besides the check against the
+    oracle, the run that the boundary splits must keep its lowest positions (Sec. 3.4 top-k,
+    ties to the lower index): identical keys have identical scores by definition."""
+    wl = W.tiny_workload(batch=2, h_q=8, h_kv=2, head_dim=128, t_ctx=4096, budget=302, n_sink=4, n_recent=32,
+                         window=32, gamma=1, seed=77 + run)
+    inp = W.make_layer(wl, 0, "cuda")
+    lo, hi = wl.n_sink, wl.t_ctx - wl.n_recent
+    mid = inp.k_cache[:, :, lo:hi]
+    first = torch.arange(hi - lo, device=mid.device) // run * run
+    mid.copy_(mid[:, :, first].clone())
+    h = host(inp)
+    run_and_check(wl, inp, h, modes=("carry",), check_steps=False, tag=f"runs of {run}")
+    t = wl.t_ctx
+    lse_ref = oracle.window_lse(h["QW"], h["K"], t)
+    st = bd.SpecStep.for_workload(wl)
+    st.select(inp.k_cache, inp.q_win, torch.from_numpy(lse_ref).float().cuda())
+    torch.cuda.synchronize()
+    n_split = 0
+    for b in range(wl.batch):
+        for kv in range(wl.h_kv):
+            kept = st.idx[b, kv, : int(st.count[b, kv])].cpu().numpy()
+            kept = kept[(kept >= lo) & (kept < hi)] - lo
+            taken = np.bincount(kept // run, minlength=(hi - lo + run - 1) // run)
+            size = np.bincount(np.arange(hi - lo) // run)
+            for r in np.nonzero((taken > 0) & (taken < size))[0]:
+                assert np.array_equal(np.sort(kept[kept // run == r]), r * run + np.arange(taken[r])), \
+                    f"unit ({b},{kv}) run {r}: kept {np.sort(kept[kept // run == r])[:8]} are not its lowest positions"
+                n_split += 1
+    assert n_split > 0, "no run was split by the boundary"
+
+
 @pytest.mark.parametrize("d", [64, 128])
 def test_self_mode_whole_units_per_cta(d):
     """128 (sequence, KV head) units of one 128-key tile each: every CTA of the window-LSE
