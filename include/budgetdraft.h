@@ -79,7 +79,10 @@ typedef enum bd_status {
  * launches.  Everything this header says of t_ctx holds per sequence with T_b in its
  * place.  NULL: every sequence has t_ctx.  A T_b outside [1, t_ctx] is recorded in the
  * workspace status word (BD_ERR_INVALID_ARG) and clamped into range.  With seq_lens,
- * batch * h_kv must not exceed 1024 (BD_ERR_UNSUPPORTED). */
+ * batch * h_kv must not exceed 4096, and a call whose kernel keeps a table of
+ * batch * h_kv + 1 ints in shared memory (the selection's score pass, the verify pass)
+ * reports BD_ERR_UNSUPPORTED when that table does not fit beside its tiles (the verify
+ * pass with 24 query rows per KV head holds about 2500). */
 typedef struct bd_shape {
   int32_t batch;     /* sequences                                   */
   int32_t h_q;       /* query heads                                 */

@@ -1699,6 +1699,10 @@ bool select_plan(const bd_shape& s, int window, int budget, int n_sink, int n_re
     plan->lse_smem_bytes = 2048 + (size_t)2 * 128 * s.head_dim * 2 + (size_t)kLStages * kSKeys * s.head_dim * 2 +
                            2 * 128 * sizeof(float2) + (s.seq_lens ? align_up((size_t)(units + 1) * 4, 16) : 0);
     plan->lse_part_bytes = max_seg > 1 ? align_up((size_t)units * max_seg * 128 * sizeof(float2), 256) : 0;
+    // a units' table too large for shared memory: the lse-only verify kernel below instead
+    plan->lse_tc = plan->lse_smem_bytes <= 227 * 1024;
+  }
+  if (plan->lse_tc) {
     plan->self_mode = true;
   } else {
     bd_shape ls = s;

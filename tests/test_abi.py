@@ -216,6 +216,9 @@ def test_check_wait_timeout_validation(lib):
 
 
 def test_seq_lens_unit_limit(lib):
-    s = shape(batch=129, h_q=64, h_kv=8)          # 1032 units
+    s = shape(batch=513, h_q=64, h_kv=8)          # 4104 units: beyond the 4096 the tables allow
     s.seq_lens = A
     assert verify(lib, s) == UNSUPPORTED
+    s = shape(batch=129, h_q=64, h_kv=8)          # 1032 units: within them
+    s.seq_lens = A
+    assert verify(lib, s) != UNSUPPORTED

@@ -181,3 +181,60 @@ def test_ragged_multistep_each_sequence_advances_by_its_own_count():
                          - oracle.window_lse(qh[i:i + 1, :, t - W: t], Kh[i:i + 1], t)[0]).max()
             assert err <= 1e-3, f"step {step} seq {i}: slid window LSE off by {err}"
         assert ws.status() == 0
+
+
+@pytest.mark.parametrize("mode", ["carry", "self"])
+def test_ragged_mha_batch_beyond_1024_units(mode):
+    """The paper's verifier is multi-head (one query head per KV head: 32 KV heads at d 128),
+    so a ragged batch of 40 sequences already holds 1280 (sequence, KV head) units, more than
+    a table of 1024 would: selection, a draft pass and the verify, each against the oracle
+    on a sample of sequences at their own lengths."""
+    b, hq, hkv, d, W, gamma, budget, sink, recent = 40, 32, 32, 128, 32, 3, 128, 4, 16
+    g = torch.Generator().manual_seed(40)
+    lens = torch.randint(300, 901, (b,), generator=g).tolist()
+    lens[-1] = 100                                   # fits the budget: keep all
+    t_max = max(lens)
+    wl = wk.tiny_workload(batch=b, h_q=hq, h_kv=hkv, head_dim=d, t_ctx=t_max, budget=budget, n_sink=sink,
+                         n_recent=recent, window=W, gamma=gamma)
+    inp = wk.make_layer(wl, 0, "cuda")
+    lens_d = torch.tensor(lens, dtype=torch.int32, device="cuda")
+    shape = bd.make_shape(b, hq, hkv, d, t_max, wl.t_cap, seq_lens=lens_d)
+    sample = [0, 7, 19, 33, b - 1]
+    h = {i: dict(K=f64(inp.k_cache[i:i + 1]), V=f64(inp.v_cache[i:i + 1]), QW=f64(inp.q_win[i:i + 1]),
+                 QD=f64(inp.q_draft[:, i:i + 1]), QV=f64(inp.q_verify[i:i + 1])) for i in sample}
+    lse_ref = {i: oracle.window_lse(h[i]["QW"], h[i]["K"], lens[i]) for i in sample}
+    if mode == "carry":   # the carried LSE of the unsampled sequences comes from the library's own pass
+        st = bd.SpecStep(b, hq, hkv, d, t_max, wl.t_cap, budget, sink, recent, W, gamma, seq_lens=lens_d)
+        lse_d = st.window_lse(inp.k_cache, inp.q_win)
+        for i in sample:
+            lse_d[i:i + 1] = torch.from_numpy(lse_ref[i]).float().cuda()
+    else:
+        lse_d = None
+    ws = bd.Workspace.for_step(shape, budget, W, gamma)
+    idx = torch.empty(b, hkv, budget, dtype=torch.int32, device="cuda")
+    cnt = torch.empty(b, hkv, dtype=torch.int32, device="cuda")
+    bd.bd_select_budget(shape, inp.k_cache, inp.q_win, lse_d, W, budget, sink, recent, 1, idx, cnt, ws)
+    torch.cuda.synchronize()
+    refs = {}
+    for i in sample:
+        ir, cr, score = oracle_selection(h[i]["QW"], h[i]["K"], lse_ref[i], lens[i], budget, sink, recent)
+        refs[i] = (ir, cr)
+        check_selection(idx[i:i + 1], cnt[i:i + 1], ir, cr, score, lens[i], budget, sink, recent, 1,
+                        what=f"{mode} seq {i} T={lens[i]}")
+    assert int(cnt[b - 1, 0]) == lens[-1]
+    for i in sample:   # the drafts run on the oracle's view of the sampled sequences
+        idx[i] = torch.from_numpy(refs[i][0][0]).int().cuda()
+        cnt[i] = torch.from_numpy(refs[i][1][0]).int().cuda()
+    o = torch.empty(b, hq, d, dtype=torch.bfloat16, device="cuda")
+    l = torch.empty(b, hq, dtype=torch.float32, device="cuda")
+    bd.bd_draft_attn(shape, inp.q_draft[1], inp.k_cache, inp.v_cache, idx, cnt, budget, 1, o, l, ws)
+    vo = torch.empty(b, hq, gamma + 1, d, dtype=torch.bfloat16, device="cuda")
+    vl = torch.empty(b, hq, gamma + 1, dtype=torch.float32, device="cuda")
+    bd.bd_verify_attn(shape, inp.q_verify, gamma + 1, inp.k_cache, inp.v_cache, vo, vl, ws)
+    torch.cuda.synchronize()
+    for i in sample:
+        o_ref, l_ref = oracle.draft_attn(h[i]["QD"][1], h[i]["K"], h[i]["V"], refs[i][0], refs[i][1], lens[i], 1)
+        check_attention(o[i:i + 1], l[i:i + 1], o_ref, l_ref, f"{mode} draft seq {i} T={lens[i]}")
+        o_ref, l_ref = oracle.verify_attn(h[i]["QV"], h[i]["K"], h[i]["V"], lens[i])
+        check_attention(vo[i:i + 1], vl[i:i + 1], o_ref, l_ref, f"{mode} verify seq {i} T={lens[i]}")
+    assert ws.status() == 0
