@@ -45,6 +45,10 @@ cudaError_t launch_kernel(const void* fn, dim3 grid, dim3 block, size_t smem, cu
   return cudaLaunchKernelExC(&cfg, fn, args);
 }
 
+// batch * h_kv with per-sequence lengths: the score, window-LSE and verify kernels keep a
+// table of units + 1 ints in shared memory (each plan also checks that its table fits)
+constexpr int kMaxRaggedUnits = 4096;
+
 size_t ws_counters_offset() { return kWsHeaderBytes; }
 size_t ws_region_offset(int units) { return kWsHeaderBytes + align_up((size_t)units * 4, 256); }
 

@@ -24,7 +24,6 @@ struct WsHeader {          // first 256 bytes of every workspace
   int pad[63];
 };
 constexpr size_t kWsHeaderBytes = 256;
-constexpr int kMaxRaggedUnits = 4096;   // batch * h_kv with per-sequence lengths (shared-memory tables)
 
 __host__ __device__ constexpr size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
