@@ -797,12 +797,20 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_kernel(const TopkParams 
     a = max(c * s, lo);
     b = min(c * s + s, hi);
   };
+  // a chunk's score: its members summed in position order, their loads issued eight at a
+  // time (all in flight together; the zeros past b add nothing to a sum of scores >= +0)
   auto value_global = [&](int i) -> uint32_t {
     if (s == 1) return __float_as_uint(__ldcg(sc + i));
     int a, b;
     members(i, a, b);
     float v = 0.f;
-    for (int q = a; q < b; ++q) v += __ldcg(sc + (q - lo));
+    for (int q0 = a; q0 < b; q0 += 8) {
+      float t[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) t[j] = q0 + j < b ? __ldcg(sc + (q0 + j - lo)) : 0.f;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) v += t[j];
+    }
     return __float_as_uint(v);
   };
   if (ranked && staged) {
@@ -818,7 +826,14 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_kernel(const TopkParams 
       }
       for (int i = 4 * n4 + tid; i < n_items; i += kTopkThreads) vals[i] = __float_as_uint(__ldcg(sc + i));
     } else {
-      for (int i = tid; i < n_items; i += kTopkThreads) vals[i] = value_global(i);
+      // two chunks per round, so that both chunks' loads are in flight together
+      for (int i = tid; i < n_items; i += 2 * kTopkThreads) {
+        const int i2 = i + kTopkThreads;
+        const uint32_t v1 = value_global(i);
+        const uint32_t v2 = i2 < n_items ? value_global(i2) : 0u;
+        vals[i] = v1;
+        if (i2 < n_items) vals[i2] = v2;
+      }
     }
     __syncthreads();
   }
