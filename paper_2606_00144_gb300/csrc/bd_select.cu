@@ -1361,60 +1361,50 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_token_kernel(const TopkP
   if (tid == 0) p.count_out[unit] = count;
 }
 
-// Token-level selection with every score held in registers (up to 16 per thread): the same
-// boundary-bin method as topk_token_kernel with the passes unrolled at compile time over
-// the thread's ROWS items, so no pass goes through shared memory but the histogram.  Warp w
-// owns items [w*ROWS*32, (w+1)*ROWS*32), row r of it at w*ROWS*32 + 32r + lane.  Needs
-// 0 < k < n <= ROWS * kTopkThreads.
-template <int ROWS>
-__global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkParams p) {
-  __shared__ uint32_t bins[kBins];
-  __shared__ uint64_t cand[kBinCandMax];
-  __shared__ uint32_t wsum[32];
-  __shared__ float wmin[32], wmax[32];
-  __shared__ uint32_t s_total, s_bin, s_above, s_nc, s_taukey, s_eq_take, s_eq_all, s_prefix, s_krem;
-  grid_dependency_wait();
-  allow_dependent_launch();
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int unit = blockIdx.x;
-  const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
-  int32_t* out = p.idx_out + (size_t)unit * p.budget;
-  if (topk_keep_all(p, unit, t_u, out)) return;
-  const int lo = p.n_sink, hi = t_u - p.n_recent, n = hi - lo;
-  const int k = p.budget - p.n_sink - p.n_recent;
-  const float* sc = p.score + (size_t)unit * p.n_mid_pad;
-  const int w0 = warp * ROWS * 32;
+// Shared storage of the register-resident top-B kernels.
+struct TopkRowsSmem {
+  uint32_t bins[kBins];
+  uint64_t cand[kBinCandMax];
+  uint32_t wsum[32], wpos[32];
+  float wmin[32], wmax[32];
+  uint32_t s_total, s_bin, s_above, s_nc, s_taukey, s_eq_take, s_eq_all, s_prefix, s_krem;
+};
 
-  // ---- the thread's scores (fp32 bits; non-negative, so their order is the bits' order).
-  // Slots past n hold +0: no score is below it and ties go to the lower position, so the
-  // padding never displaces a real score and needs no test in the passes below.
-  uint32_t u[ROWS];
-  float lmin = INFINITY, lmax = -INFINITY;
-#pragma unroll
-  for (int r = 0; r < ROWS; ++r) {
-    const int i = w0 + 32 * r + lane;
-    const float v = i < n ? __ldcg(sc + i) : 0.f;
-    u[r] = __float_as_uint(v);
-    lmin = fminf(lmin, v);
-    lmax = fmaxf(lmax, v);
-  }
-  for (int i = tid; i < kBins; i += kTopkThreads) bins[i] = 0;
+// The k-th largest of the block's items: tau (its fp32 bits), krem (how many items equal to
+// tau are kept, in item order) and whether that is all of them.
+struct RowsThreshold {
+  uint32_t tau, krem;
+  bool simple;
+};
+
+// Items in registers, ROWS per thread: warp w owns items [w*ROWS*32, (w+1)*ROWS*32), row r of
+// it at w*ROWS*32 + 32r + lane; values are fp32 bits of non-negative scores (the order of the
+// bits), +0 in slots past the item count (no item is below it and ties go to the lower item,
+// so the padding never displaces an item).  A linear histogram between the smallest and the
+// largest value (lmin, lmax: this thread's) finds the bin of the k-th value and its items are
+// ranked exactly; a crowded bin takes an exact 4-pass radix select on the bits.  0 < k < n.
+template <int ROWS>
+__device__ __forceinline__ RowsThreshold rows_threshold(TopkRowsSmem& S, const uint32_t (&u)[ROWS], float lmin,
+                                                        float lmax, int k) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int w0 = warp * ROWS * 32;
+  for (int i = tid; i < kBins; i += kTopkThreads) S.bins[i] = 0;
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     lmin = fminf(lmin, __shfl_xor_sync(0xffffffffu, lmin, off));
     lmax = fmaxf(lmax, __shfl_xor_sync(0xffffffffu, lmax, off));
   }
   if (lane == 0) {
-    wmin[warp] = lmin;
-    wmax[warp] = lmax;
+    S.wmin[warp] = lmin;
+    S.wmax[warp] = lmax;
   }
   if (tid == 0) {
-    s_nc = 0;
-    s_eq_take = 0;
-    s_eq_all = 0;
+    S.s_nc = 0;
+    S.s_eq_take = 0;
+    S.s_eq_all = 0;
   }
   __syncthreads();
-  float vmin = wmin[lane], vmax = wmax[lane];
+  float vmin = S.wmin[lane], vmax = S.wmax[lane];
 #pragma unroll
   for (int off = 16; off > 0; off >>= 1) {
     vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, off));
@@ -1428,11 +1418,11 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     const float scale = (float)(kBins - 1) / (vmax - vmin);
     auto bin_of = [&](uint32_t x) -> int { return min(kBins - 1, (int)((__uint_as_float(x) - vmin) * scale)); };
 #pragma unroll
-    for (int r = 0; r < ROWS; ++r) atomicAdd(&bins[bin_of(u[r])], 1u);
+    for (int r = 0; r < ROWS; ++r) atomicAdd(&S.bins[bin_of(u[r])], 1u);
     __syncthreads();
     constexpr int BPT = kBins / kTopkThreads;
     uint32_t hb[BPT];
-    const uint4 hv = reinterpret_cast<const uint4*>(bins)[tid];
+    const uint4 hv = reinterpret_cast<const uint4*>(S.bins)[tid];
     hb[0] = hv.x;
     hb[1] = hv.y;
     hb[2] = hv.z;
@@ -1443,61 +1433,61 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
       const uint32_t z = __shfl_up_sync(0xffffffffu, incl, off);
       if (lane >= off) incl += z;
     }
-    if (lane == 31) wsum[warp] = incl;
+    if (lane == 31) S.wsum[warp] = incl;
     __syncthreads();
     if (warp == 0) {
-      const uint32_t w = wsum[lane];
+      const uint32_t w = S.wsum[lane];
       uint32_t c = w;
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
         const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
         if (lane >= off) c += z;
       }
-      wsum[lane] = c - w;
-      if (lane == 31) s_total = c;
+      S.wsum[lane] = c - w;
+      if (lane == 31) S.s_total = c;
     }
     __syncthreads();
-    uint32_t above = s_total - (wsum[warp] + incl);
+    uint32_t above = S.s_total - (S.wsum[warp] + incl);
 #pragma unroll
     for (int j = BPT - 1; j >= 0; --j) {
       if (above < (uint32_t)k && (uint32_t)k <= above + hb[j]) {
-        s_bin = (uint32_t)(tid * BPT + j);
-        s_above = above;
-        s_prefix = hb[j];
+        S.s_bin = (uint32_t)(tid * BPT + j);
+        S.s_above = above;
+        S.s_prefix = hb[j];
       }
       above += hb[j];
     }
     __syncthreads();
-    const int bstar = (int)s_bin;
-    const uint32_t nc = s_prefix;
+    const int bstar = (int)S.s_bin;
+    const uint32_t nc = S.s_prefix;
     if (nc <= (uint32_t)kBinCandMax) {
 #pragma unroll
       for (int r = 0; r < ROWS; ++r) {
         const int i = w0 + 32 * r + lane;
         if (bin_of(u[r]) == bstar)
-          cand[atomicAdd(&s_nc, 1u)] = (static_cast<uint64_t>(u[r]) << 32) | (0xFFFFFFFFu - (uint32_t)i);
+          S.cand[atomicAdd(&S.s_nc, 1u)] = (static_cast<uint64_t>(u[r]) << 32) | (0xFFFFFFFFu - (uint32_t)i);
       }
       __syncthreads();
-      const uint32_t m = (uint32_t)k - s_above;
+      const uint32_t m = (uint32_t)k - S.s_above;
       for (int i = tid; i < (int)nc; i += kTopkThreads) {
-        const uint64_t kk = cand[i];
+        const uint64_t kk = S.cand[i];
         uint32_t rk = 0;
-        for (int j = 0; j < (int)nc; ++j) rk += cand[j] > kk;
-        if (rk == m - 1) s_taukey = static_cast<uint32_t>(kk >> 32);
+        for (int j = 0; j < (int)nc; ++j) rk += S.cand[j] > kk;
+        if (rk == m - 1) S.s_taukey = static_cast<uint32_t>(kk >> 32);
       }
       __syncthreads();
-      tau = s_taukey;
+      tau = S.s_taukey;
       for (int i = tid; i < (int)nc; i += kTopkThreads) {
-        const uint64_t kk = cand[i];
+        const uint64_t kk = S.cand[i];
         if (static_cast<uint32_t>(kk >> 32) != tau) continue;
         uint32_t rk = 0;
-        for (int j = 0; j < (int)nc; ++j) rk += cand[j] > kk;
-        atomicAdd(&s_eq_all, 1u);
-        if (rk < m) atomicAdd(&s_eq_take, 1u);
+        for (int j = 0; j < (int)nc; ++j) rk += S.cand[j] > kk;
+        atomicAdd(&S.s_eq_all, 1u);
+        if (rk < m) atomicAdd(&S.s_eq_take, 1u);
       }
       __syncthreads();
-      krem = s_eq_take;
-      simple = (s_eq_take == s_eq_all);
+      krem = S.s_eq_take;
+      simple = (S.s_eq_take == S.s_eq_all);
       found = true;
     }
   }
@@ -1507,16 +1497,16 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     krem = (uint32_t)k;
     for (int pass = 0; pass < 4; ++pass) {
       const int shift = 24 - 8 * pass;
-      for (int i = tid; i < 256; i += kTopkThreads) bins[i] = 0;
+      for (int i = tid; i < 256; i += kTopkThreads) S.bins[i] = 0;
       __syncthreads();
 #pragma unroll
       for (int r = 0; r < ROWS; ++r)
-        if ((u[r] & mask) == prefix) atomicAdd(&bins[(u[r] >> shift) & 255u], 1u);
+        if ((u[r] & mask) == prefix) atomicAdd(&S.bins[(u[r] >> shift) & 255u], 1u);
       __syncthreads();
       if (warp == 0) {
         uint32_t local = 0;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) local += bins[8 * lane + j];
+        for (int j = 0; j < 8; ++j) local += S.bins[8 * lane + j];
         uint32_t suffix = local;
 #pragma unroll
         for (int off = 1; off < 32; off <<= 1) {
@@ -1526,10 +1516,10 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
         uint32_t abv = suffix - local;
         if (abv < krem && krem <= suffix) {
           for (int j = 7; j >= 0; --j) {
-            const uint32_t h = bins[8 * lane + j];
+            const uint32_t h = S.bins[8 * lane + j];
             if (abv + h >= krem) {
-              s_prefix = prefix | ((uint32_t)(8 * lane + j) << shift);
-              s_krem = krem - abv;
+              S.s_prefix = prefix | ((uint32_t)(8 * lane + j) << shift);
+              S.s_krem = krem - abv;
               break;
             }
             abv += h;
@@ -1537,14 +1527,26 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
         }
       }
       __syncthreads();
-      prefix = s_prefix;
-      krem = s_krem;
+      prefix = S.s_prefix;
+      krem = S.s_krem;
       mask |= 0xFFu << shift;
     }
     tau = prefix;
     simple = false;
   }
 
+  return RowsThreshold{tau, krem, simple};
+}
+
+// Ascending compaction of the kept items (warp ballots, a block scan, the writes), then the
+// sinks, the recent window and the padding: the token-level output.
+template <int ROWS>
+__device__ __forceinline__ void rows_compact_tokens(TopkRowsSmem& S, const uint32_t (&u)[ROWS], RowsThreshold th,
+                                                    const TopkParams& p, int unit, int lo, int hi, int32_t* out) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int w0 = warp * ROWS * 32;
+  const uint32_t tau = th.tau, krem = th.krem;
+  const bool simple = th.simple;
   // ---- ascending compaction: warp ballots of the selected items, block scan, writes
   const uint32_t lt = (1u << lane) - 1u;
   uint32_t eq_base = 0;
@@ -1554,20 +1556,20 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
 #pragma unroll
     for (int r = 0; r < ROWS; ++r)
       eqc += __popc(__ballot_sync(0xffffffffu, u[r] == tau));
-    if (lane == 0) wsum[warp] = eqc;
+    if (lane == 0) S.wsum[warp] = eqc;
     __syncthreads();
     if (warp == 0) {
-      const uint32_t w = wsum[lane];
+      const uint32_t w = S.wsum[lane];
       uint32_t c = w;
 #pragma unroll
       for (int off = 1; off < 32; off <<= 1) {
         const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
         if (lane >= off) c += z;
       }
-      wsum[lane] = c - w;
+      S.wsum[lane] = c - w;
     }
     __syncthreads();
-    eq_base = wsum[warp];
+    eq_base = S.wsum[warp];
     __syncthreads();
   }
   uint32_t masks[ROWS];
@@ -1586,21 +1588,21 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     masks[r] = __ballot_sync(0xffffffffu, sel);
     cnt += __popc(masks[r]);
   }
-  if (lane == 0) wsum[warp] = cnt;
+  if (lane == 0) S.wsum[warp] = cnt;
   __syncthreads();
   if (warp == 0) {
-    const uint32_t w = wsum[lane];
+    const uint32_t w = S.wsum[lane];
     uint32_t c = w;
 #pragma unroll
     for (int off = 1; off < 32; off <<= 1) {
       const uint32_t z = __shfl_up_sync(0xffffffffu, c, off);
       if (lane >= off) c += z;
     }
-    wsum[lane] = c - w;
-    if (lane == 31) s_total = c;
+    S.wsum[lane] = c - w;
+    if (lane == 31) S.s_total = c;
   }
   __syncthreads();
-  uint32_t base = (uint32_t)lo + wsum[warp];
+  uint32_t base = (uint32_t)lo + S.wsum[warp];
 #pragma unroll
   for (int r = 0; r < ROWS; ++r) {
     const uint32_t mk = masks[r];
@@ -1608,7 +1610,164 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
     if ((mk >> lane) & 1u) out[base + __popc(mk & lt)] = lo + w0 + 32 * r + lane;
     base += __popc(mk);
   }
-  const int n_chosen = (int)s_total;
+  const int n_chosen = (int)S.s_total;
+  const int count = lo + n_chosen + p.n_recent;
+  for (int i = tid; i < lo; i += kTopkThreads) out[i] = i;
+  for (int i = tid; i < p.n_recent; i += kTopkThreads) out[lo + n_chosen + i] = hi + i;
+  for (int i = count + tid; i < p.budget; i += kTopkThreads) out[i] = -1;
+  if (tid == 0) p.count_out[unit] = count;
+}
+
+// Token-level selection with every score held in registers (up to 16 per thread), the count
+// a template parameter so every pass is straight-line code.  Needs 0 < k < n <= ROWS * kTopkThreads.
+template <int ROWS>
+__global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkParams p) {
+  __shared__ TopkRowsSmem S;
+  grid_dependency_wait();
+  allow_dependent_launch();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int unit = blockIdx.x;
+  const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
+  int32_t* out = p.idx_out + (size_t)unit * p.budget;
+  if (topk_keep_all(p, unit, t_u, out)) return;
+  const int lo = p.n_sink, hi = t_u - p.n_recent, n = hi - lo;
+  const int k = p.budget - p.n_sink - p.n_recent;
+  const float* sc = p.score + (size_t)unit * p.n_mid_pad;
+  const int w0 = warp * ROWS * 32;
+  uint32_t u[ROWS];
+  float lmin = INFINITY, lmax = -INFINITY;
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    const int i = w0 + 32 * r + lane;
+    const float v = i < n ? __ldcg(sc + i) : 0.f;
+    u[r] = __float_as_uint(v);
+    lmin = fminf(lmin, v);
+    lmax = fmaxf(lmax, v);
+  }
+  rows_compact_tokens<ROWS>(S, u, rows_threshold<ROWS>(S, u, lmin, lmax, k), p, unit, lo, hi, out);
+}
+
+// Chunk-level selection (chunk = s > 1, the paper's policy) with every chunk's score in
+// registers.  Chunk c covers positions [c s, c s + s) clipped to the middle [lo, hi), so the
+// first and the last may hold fewer, and scores the sum of its members' scores in position
+// order; the top k = floor(free / s) chunks (ties to the lower chunk) by rows_threshold are
+// written member by member in position order.  Items are the chunks, n_items <= ROWS *
+// kTopkThreads; a unit with no chunk to rank keeps all of them or none.
+template <int ROWS>
+__global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_chunk_kernel(const TopkParams p) {
+  __shared__ TopkRowsSmem S;
+  grid_dependency_wait();
+  allow_dependent_launch();
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int unit = blockIdx.x;
+  const int t_u = unit_context(p.seq_lens, unit, p.h_kv, p.t_ctx, tid == 0 ? p.status : nullptr);
+  int32_t* out = p.idx_out + (size_t)unit * p.budget;
+  if (topk_keep_all(p, unit, t_u, out)) return;
+  const int lo = p.n_sink, hi = t_u - p.n_recent, s = p.chunk;
+  const int c_first = lo / s;
+  const int n_items = hi > lo ? (hi - 1) / s - c_first + 1 : 0;
+  const int k = min((p.budget - p.n_sink - p.n_recent) / s, n_items);
+  const bool take_all = k >= n_items, ranked = k > 0 && !take_all;
+  const float* sc = p.score + (size_t)unit * p.n_mid_pad;
+  const int w0 = warp * ROWS * 32;
+  auto members = [&](int i, int& a, int& b) {
+    const int c = c_first + i;
+    a = max(c * s, lo);
+    b = min(c * s + s, hi);
+  };
+
+  // ---- chunk scores: members summed in position order, their loads eight at a time (four
+  // rows' chunks in flight together; the zeros past b add nothing to scores >= +0)
+  constexpr int RB = ROWS < 4 ? ROWS : 4;
+  uint32_t u[ROWS];
+  float lmin = INFINITY, lmax = -INFINITY;
+#pragma unroll
+  for (int r0 = 0; r0 < ROWS; r0 += RB) {
+    int ma[RB], mb[RB];
+    float v[RB];
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      const int i = w0 + 32 * (r0 + r) + lane;
+      ma[r] = 0;
+      mb[r] = 0;
+      if (i < n_items) members(i, ma[r], mb[r]);
+      v[r] = 0.f;
+    }
+    for (int q0 = 0; q0 < s; q0 += 8) {
+      float t[RB][8];
+#pragma unroll
+      for (int r = 0; r < RB; ++r)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int q = ma[r] + q0 + j;
+          t[r][j] = q < mb[r] ? __ldcg(sc + (q - lo)) : 0.f;
+        }
+#pragma unroll
+      for (int r = 0; r < RB; ++r)
+#pragma unroll
+        for (int j = 0; j < 8; ++j) v[r] += t[r][j];
+    }
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      u[r0 + r] = __float_as_uint(v[r]);            // +0 past n_items
+      lmin = fminf(lmin, v[r]);
+      lmax = fmaxf(lmax, v[r]);
+    }
+  }
+  RowsThreshold th{0u, 0u, true};
+  if (ranked) th = rows_threshold<ROWS>(S, u, lmin, lmax, k);
+
+  // ---- kept chunks, their members in position order
+  const uint32_t lt = (1u << lane) - 1u;
+  uint32_t eq_base = 0;
+  if (ranked && !th.simple) {   // chunks equal to tau are taken in chunk order: those before this warp
+    uint32_t eqc = 0;
+#pragma unroll
+    for (int r = 0; r < ROWS; ++r) eqc += __popc(__ballot_sync(0xffffffffu, w0 + 32 * r + lane < n_items && u[r] == th.tau));
+    if (lane == 0) S.wsum[warp] = eqc;
+    __syncthreads();
+    eq_base = __reduce_add_sync(0xffffffffu, lane < warp ? S.wsum[lane] : 0u);
+    __syncthreads();
+  }
+  bool sel[ROWS];
+  int incl[ROWS], rowoff[ROWS];
+  int warp_pos = 0;
+  uint32_t eq_run = eq_base;
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    const bool real = w0 + 32 * r + lane < n_items;
+    bool sl = real && (take_all || (ranked && u[r] > th.tau));
+    const bool eq = real && ranked && u[r] == th.tau;
+    const uint32_t be = __ballot_sync(0xffffffffu, eq);
+    if (eq) sl = th.simple || eq_run + __popc(be & lt) < th.krem;
+    eq_run += __popc(be);
+    sel[r] = sl;
+    int a = 0, b = 0;
+    if (real) members(w0 + 32 * r + lane, a, b);
+    const int m = sl ? b - a : 0;
+    int c = m;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, c, off);
+      if (lane >= off) c += y;
+    }
+    incl[r] = c;
+    rowoff[r] = warp_pos;
+    warp_pos += __shfl_sync(0xffffffffu, c, 31);
+  }
+  if (lane == 0) S.wpos[warp] = (uint32_t)warp_pos;
+  __syncthreads();
+  const int base = lo + (int)__reduce_add_sync(0xffffffffu, lane < warp ? S.wpos[lane] : 0u);
+  const int n_chosen = (int)__reduce_add_sync(0xffffffffu, S.wpos[lane]);
+#pragma unroll
+  for (int r = 0; r < ROWS; ++r) {
+    if (sel[r]) {
+      int a, b;
+      members(w0 + 32 * r + lane, a, b);
+      int o = base + rowoff[r] + incl[r] - (b - a);
+      for (int q = a; q < b; ++q) out[o++] = q;
+    }
+  }
   const int count = lo + n_chosen + p.n_recent;
   for (int i = tid; i < lo; i += kTopkThreads) out[i] = i;
   for (int i = tid; i < p.n_recent; i += kTopkThreads) out[lo + n_chosen + i] = hi + i;
@@ -1853,6 +2012,20 @@ cudaError_t launch_select(const bd_shape& s, const SelectPlan& plan, const void*
     err = cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (err != cudaSuccess) return err;
     return launch_kernel(fn, dim3(units), dim3(kTopkThreads), smem, stream, targs, 0);
+  }
+  if (!plan.keep_all && plan.need_scores && chunk > 1) {
+    // chunks of the longest middle: the register kernel while it holds them
+    const int lo = n_sink, hi = s.t_ctx - n_recent;
+    const int n_items = hi > lo ? (hi - 1) / chunk - lo / chunk + 1 : 0;
+    if (n_items <= 16 * kTopkThreads) {
+      const int rows = std::max(1, (n_items + kTopkThreads - 1) / kTopkThreads);
+      void* fn = rows <= 1   ? reinterpret_cast<void*>(&topk_rows_chunk_kernel<1>)
+                 : rows <= 2 ? reinterpret_cast<void*>(&topk_rows_chunk_kernel<2>)
+                 : rows <= 4 ? reinterpret_cast<void*>(&topk_rows_chunk_kernel<4>)
+                 : rows <= 8 ? reinterpret_cast<void*>(&topk_rows_chunk_kernel<8>)
+                             : reinterpret_cast<void*>(&topk_rows_chunk_kernel<16>);
+      return launch_kernel(fn, dim3(units), dim3(kTopkThreads), 0, stream, targs, 0);
+    }
   }
   const int extra = kBins * 4 + kBinCandMax * 8 + 16;      // histogram + boundary-bin candidates
   const int max_items = (kTopkSmemBytes - extra) / 4;
