@@ -21,10 +21,11 @@
 //               max score finds the bin holding the k-th largest; that bin's few items are
 //               ranked exactly by (score desc, position asc) (4-pass radix select on the
 //               fp32 bits when the bin is crowded); then an ascending compaction (warp
-//               ballots + block scan) with sinks and recents.  Three kernels of that
+//               ballots + block scan) with sinks and recents.  Four kernels of that
 //               method: topk_rows_kernel (token level, up to 16K middle positions, every
-//               score in registers), topk_token_kernel (token level, up to 32K, scores in
-//               shared memory) and topk_kernel (chunk level and longer contexts).
+//               score in registers), topk_rows_chunk_kernel (chunk level, up to 16K chunks,
+//               every chunk score in registers), topk_token_kernel (token level, up to 32K,
+//               scores in shared memory) and topk_kernel (longer middles of either level).
 #include <algorithm>
 
 #include "bd_common.cuh"
