@@ -1624,6 +1624,9 @@ __device__ __forceinline__ void rows_compact_tokens(TopkRowsSmem& S, const uint3
 template <int ROWS>
 __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkParams p) {
   __shared__ TopkRowsSmem S;
+  // the unit's scores on their way into L2 while the score kernel finishes (its K stream
+  // has pushed the early ones out to DRAM by now)
+  prefetch_lines_l2(p.score + (size_t)blockIdx.x * p.n_mid_pad, (size_t)p.n_mid_pad * 4, threadIdx.x, kTopkThreads);
   grid_dependency_wait();
   allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -1657,6 +1660,7 @@ __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_kernel(const TopkPa
 template <int ROWS>
 __global__ void __launch_bounds__(kTopkThreads, 1) topk_rows_chunk_kernel(const TopkParams p) {
   __shared__ TopkRowsSmem S;
+  prefetch_lines_l2(p.score + (size_t)blockIdx.x * p.n_mid_pad, (size_t)p.n_mid_pad * 4, threadIdx.x, kTopkThreads);
   grid_dependency_wait();
   allow_dependent_launch();
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
