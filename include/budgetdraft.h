@@ -172,7 +172,7 @@ enum {
  *            with 0 <= count <= budget.
  *   flags    0 or BD_DRAFT_VIEW_READY.
  *   o_out    bf16 [batch, h_q, d];  lse_out fp32 [batch, h_q] (may be NULL).
- * Constraints: step_j >= 0, t_ctx + step_j < t_cap, h_q / h_kv <= 8.
+ * Constraints: step_j >= 0, t_ctx + step_j < t_cap, h_q / h_kv <= 16.
  */
 int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
                   const int32_t* idx, const int32_t* count, int budget, int step_j, unsigned flags,

@@ -125,7 +125,7 @@ int* status_word(void* ws) { return static_cast<int*>(ws); }
 int* counters(void* ws) { return reinterpret_cast<int*>(static_cast<uint8_t*>(ws) + ws_counters_offset()); }
 void* region(void* ws, int units) { return static_cast<uint8_t*>(ws) + ws_region_offset(units); }
 
-bool group_supported_by_draft(int g) { return g >= 1 && g <= 8; }
+bool group_supported_by_draft(int g) { return g >= 1 && g <= 16; }
 
 size_t verify_ws(const bd_shape& s, int n_q, bool with_v, bool* ok) {
   VerifyPlan vp;

@@ -9,7 +9,7 @@
 //   2. rows (80 per CTA) are gathered with 16-byte cp.async straight into the 128-byte
 //      swizzled layout (unused rows zero-filled) and the five warps run the mma.sync
 //      sub-tile code shared with the verify kernel (bd_attn_warp.cuh), the G heads of the
-//      GQA group forming one n8 query tile;
+//      GQA group forming one n8 query tile (two for groups of 9 to 16);
 //   3. every CTA stores its normalised partial straight into the shared memory of the
 //      cluster's rank-0 CTA (distributed shared memory); after one cluster barrier rank 0
 //      merges them (log-sum-exp) from its own shared memory and writes the bf16 output:
@@ -57,9 +57,10 @@ struct DraftParams {
 
 template <int D, int G>
 struct DraftSmem {
+  static constexpr int NQC = 8 * ((G + 7) / 8);   // query columns: the group in n8 tiles
   static constexpr uint32_t TILE_BYTES = kDRows * D * 2;
   static constexpr uint32_t STAGE_BYTES = 2 * TILE_BYTES;                 // K and V
-  static constexpr size_t kMerge = (size_t)(3 * kDWarps * 8) * 4 + (size_t)kDWarps * 8 * (D + 4) * 4;
+  static constexpr size_t kMerge = (size_t)(3 * kDWarps * NQC) * 4 + (size_t)kDWarps * NQC * (D + 4) * 4;
   // one CTA's partial in rank 0: G rows of D floats, then G lse padded to 16 bytes
   static constexpr int kSlot = G * D + ((G + 3) & ~3);
   // stages (the warp-merge scratch reuses them) | rowpos [pos_slots] (the row of every
@@ -73,6 +74,7 @@ struct DraftSmem {
 template <int D, int G>
 __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   using L = DraftSmem<D, G>;
+  constexpr int NT = (G + 7) / 8, NQC = L::NQC;   // the group's query heads in n8 tiles
   constexpr uint32_t HALF_BYTES = kDRows * 128;
   constexpr int CH = D / 8;                    // 16-byte chunks per row
   const bool early = (p.flags & BD_DRAFT_VIEW_READY) != 0;
@@ -92,9 +94,9 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   int* rowpos = reinterpret_cast<int*>(smem + stage_bytes);               // [pos_slots]
   float* parts = reinterpret_cast<float*>(rowpos + p.pos_slots);          // [C][kSlot]
   float* m_s = reinterpret_cast<float*>(stage);                           // warp-merge scratch
-  float* l_s = m_s + kDWarps * 8;
-  float* f_s = l_s + kDWarps * 8;
-  float* o_s = f_s + kDWarps * 8;
+  float* l_s = m_s + kDWarps * NQC;
+  float* f_s = l_s + kDWarps * NQC;
+  float* o_s = f_s + kDWarps * NQC;
 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int split = blockIdx.x, unit = blockIdx.y;
@@ -170,9 +172,9 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     allow_dependent_launch();
     if (n_tiles > 0) gather(0, 0, 1);
   }
-  uint32_t bq[1][D / 16][2];
-  WarpAttn<D, 1, true>::load_q(bq, p.q + (size_t)unit * p.g * D, p.g, 0, lane);
-  WarpAttn<D, 1, true> wa;
+  uint32_t bq[NT][D / 16][2];
+  WarpAttn<D, NT, true>::load_q(bq, p.q + (size_t)unit * p.g * D, p.g, 0, lane);
+  WarpAttn<D, NT, true> wa;
   wa.init();
   for (int t = 0; t < n_tiles; ++t) {
     const int b = dbuf ? (t & 1) : 0;
@@ -197,11 +199,11 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
     if (!dbuf && t + 1 < n_tiles) gather(t + 1, 0, 2);
   }
   wa.finish_rows();
-  wa.store(m_s, l_s, o_s, warp, 8, 0, lane);
+  wa.store(m_s, l_s, o_s, warp, NQC, 0, lane);
   __syncthreads();
   const size_t row0 = (size_t)unit * p.g;
   if (p.n_split == 1) {
-    merge_warps_flat<D, kDWarps, true>(m_s, l_s, o_s, 8, p.g, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D, tid,
+    merge_warps_flat<D, kDWarps, true>(m_s, l_s, o_s, NQC, p.g, p.lse ? p.lse + row0 : nullptr, p.o + row0 * D, tid,
                                        kDThreads);
     return;
   }
@@ -212,7 +214,7 @@ __global__ void __launch_bounds__(kDThreads) draft_kernel(const DraftParams p) {
   const int rank = (int)cluster.block_rank();
   float* slot = cluster.map_shared_rank(parts, 0) + (size_t)rank * SLOT;   // in rank 0
   asm volatile("barrier.cluster.wait.aligned;" ::: "memory");          // every CTA is running
-  merge_warps_flat<D, kDWarps, false>(m_s, l_s, o_s, 8, G, slot + G * D, slot, tid, kDThreads);
+  merge_warps_flat<D, kDWarps, false>(m_s, l_s, o_s, NQC, G, slot + G * D, slot, tid, kDThreads);
   cluster.sync();                                  // all partials have landed in rank 0
   if (rank != 0) return;
   // each thread: four output columns of one head, its merge weights derived in place
@@ -255,27 +257,28 @@ using DraftFn = void*;
 DraftFn pick(int d, int g) {
 #define BD_DK(DD, GG) \
   if (d == DD && g == GG) return reinterpret_cast<void*>(&draft_kernel<DD, GG>);
-  BD_DK(64, 1) BD_DK(64, 2) BD_DK(64, 4) BD_DK(64, 8)
-  BD_DK(128, 1) BD_DK(128, 2) BD_DK(128, 4) BD_DK(128, 8)
+  BD_DK(64, 1) BD_DK(64, 2) BD_DK(64, 4) BD_DK(64, 8) BD_DK(64, 16)
+  BD_DK(128, 1) BD_DK(128, 2) BD_DK(128, 4) BD_DK(128, 8) BD_DK(128, 16)
 #undef BD_DK
   return nullptr;
 }
 size_t smem_bytes(int d, int g, int n_stage, int cluster, int pos_slots) {
 #define BD_DS(DD, GG) \
   if (d == DD && g == GG) return DraftSmem<DD, GG>::bytes(n_stage, cluster, pos_slots);
-  BD_DS(64, 1) BD_DS(64, 2) BD_DS(64, 4) BD_DS(64, 8)
-  BD_DS(128, 1) BD_DS(128, 2) BD_DS(128, 4) BD_DS(128, 8)
+  BD_DS(64, 1) BD_DS(64, 2) BD_DS(64, 4) BD_DS(64, 8) BD_DS(64, 16)
+  BD_DS(128, 1) BD_DS(128, 2) BD_DS(128, 4) BD_DS(128, 8) BD_DS(128, 16)
 #undef BD_DS
   return 0;
 }
 }  // namespace
 
-// The kernel instance whose n8 query tile holds a group of g query heads (g <= 8).
-int draft_group_instance(int g) { return g <= 1 ? 1 : g <= 2 ? 2 : g <= 4 ? 4 : 8; }
+// The kernel instance whose n8 query tiles hold a group of g query heads (g <= 16: one
+// tile up to 8, two beyond).
+int draft_group_instance(int g) { return g <= 1 ? 1 : g <= 2 ? 2 : g <= 4 ? 4 : g <= 8 ? 8 : 16; }
 
 bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
   const int g = s.h_q / s.h_kv;
-  if (g < 1 || g > 8 || !pick(s.head_dim, draft_group_instance(g))) return false;
+  if (g < 1 || g > 16 || !pick(s.head_dim, draft_group_instance(g))) return false;
   const long entries = (long)budget + n_steps;
   // one tile per CTA up to a cluster of 8, but no more CTAs than one wave holds at the
   // occupancy the slice's stage count gives (three single-stage or two double-buffered

@@ -88,7 +88,8 @@ def test_draft_validation(lib):
     assert draft(lib, shape(), j=-1) == INVALID
     assert draft(lib, shape(), j=10) == INVALID                       # t_ctx + j >= t_cap
     assert draft(lib, shape(), budget=0) == INVALID
-    assert draft(lib, shape(h_q=18, h_kv=2)) == UNSUPPORTED           # group of 9 > 8
+    assert draft(lib, shape(h_q=34, h_kv=2)) == UNSUPPORTED           # group of 17 > 16
+    assert draft(lib, shape(h_q=18, h_kv=2)) != UNSUPPORTED           # group of 9: two query tiles
     assert draft(lib, shape(), flags=6) == INVALID                    # unknown flag bits
 
 
