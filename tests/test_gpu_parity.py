@@ -437,15 +437,16 @@ def test_exact_ties_ranked_above_the_bound(run):
     assert n_split > 0, "no run was split by the boundary"
 
 
+@pytest.mark.parametrize("d", [64, 128])
 @pytest.mark.parametrize("h_q", [18, 32])
-def test_groups_beyond_one_query_tile(h_q):
+def test_groups_beyond_one_query_tile(h_q, d):
     """GQA groups of 9 and 16 query heads per KV head: the draft kernel holds the group in two
     n8 query tiles (the selection with a 16-row window keeps G * W <= 256 rows; carry mode,
     as self mode takes at most 128 window rows), checked step by step against the oracle."""
-    wl = W.tiny_workload(batch=2, h_q=h_q, h_kv=2, head_dim=128, t_ctx=900, budget=128, n_sink=4, n_recent=16,
+    wl = W.tiny_workload(batch=2, h_q=h_q, h_kv=2, head_dim=d, t_ctx=900, budget=128, n_sink=4, n_recent=16,
                          window=16, gamma=3)
     inp = W.make_layer(wl, 0, "cuda")
-    run_and_check(wl, inp, host(inp), modes=("carry",), tag=f"group {h_q // 2}")
+    run_and_check(wl, inp, host(inp), modes=("carry",), tag=f"group {h_q // 2} d{d}")
 
 
 @pytest.mark.parametrize("d", [64, 128])
