@@ -252,7 +252,7 @@ int bd_combine(const float* o_part, const float* lse_part, int n_split, int rows
  * gives 0.
  *   logits   bf16 or fp32 [rows, vocab] as `dtype` says (BD_DTYPE_*);
  *   ids_out  int32 [rows].
- * Constraints: 0 <= rows <= 65535 (0 is a no-op), vocab >= 1.  No workspace.
+ * Constraints: 0 <= rows <= 65535 (0 is a no-op), 1 <= vocab <= 2^30.  No workspace.
  */
 int bd_argmax(const void* logits, int dtype, int rows, int vocab, int32_t* ids_out, void* stream);
 

@@ -294,7 +294,9 @@ int bd_argmax(const void* logits, int dtype, int rows, int vocab, int32_t* ids_o
   if (dtype != BD_DTYPE_BF16 && dtype != BD_DTYPE_F32) return BD_ERR_INVALID_ARG;
   if (rows < 0 || vocab < 1) return BD_ERR_INVALID_ARG;
   if (rows == 0) return BD_OK;
-  if (rows > 65535) return BD_ERR_UNSUPPORTED;
+  // the kernel's element indices (a CTA's range end, a vector batch's first element) stay
+  // below 2^31 for rows of up to 2^30 elements
+  if (rows > 65535 || vocab > (1 << 30)) return BD_ERR_UNSUPPORTED;
   BD_TRY(check_tensor(logits, dtype == BD_DTYPE_BF16 ? 2 : 4));
   BD_TRY(check_tensor(ids_out, 4));
   return map_cuda(launch_argmax(logits, dtype == BD_DTYPE_BF16, rows, vocab, ids_out,

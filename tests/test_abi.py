@@ -135,6 +135,7 @@ def test_argmax_validation(lib):
     assert f(A, binding.BD_DTYPE_BF16, 4, 0, A, None) == INVALID
     assert f(A, binding.BD_DTYPE_BF16, 0, 100, A, None) == BD_OK         # empty: no-op
     assert f(A, binding.BD_DTYPE_BF16, 70000, 100, A, None) == UNSUPPORTED
+    assert f(A, binding.BD_DTYPE_BF16, 4, (1 << 30) + 1, A, None) == UNSUPPORTED   # indices past 2^31
     assert f(A + 1, binding.BD_DTYPE_BF16, 4, 100, A, None) == MISALIGNED
     assert f(A + 2, binding.BD_DTYPE_F32, 4, 100, A, None) == MISALIGNED
     assert f(A, binding.BD_DTYPE_F32, 4, 100, A + 2, None) == MISALIGNED
