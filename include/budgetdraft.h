@@ -172,7 +172,11 @@ enum {
  *            with 0 <= count <= budget.
  *   flags    0 or BD_DRAFT_VIEW_READY.
  *   o_out    bf16 [batch, h_q, d];  lse_out fp32 [batch, h_q] (may be NULL).
- * Constraints: step_j >= 0, t_ctx + step_j < t_cap, h_q / h_kv <= 16.
+ * Constraints: step_j >= 0, t_ctx + step_j < t_cap, h_q / h_kv <= 16.  The budget + step_j + 1
+ * entries are split over at most 8 CTAs, each holding the row table of its slice in shared
+ * memory beside its tiles: at head_dim 128 views of up to about 165K (GQA group 16) to
+ * 290K (group 1) entries, fewer when batch * h_kv fills the GPU; a larger view returns
+ * BD_ERR_UNSUPPORTED.
  */
 int bd_draft_attn(const bd_shape* shape, const void* q, const void* k_cache, const void* v_cache,
                   const int32_t* idx, const int32_t* count, int budget, int step_j, unsigned flags,

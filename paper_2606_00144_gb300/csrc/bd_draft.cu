@@ -272,6 +272,19 @@ size_t smem_bytes(int d, int g, int n_stage, int cluster, int pos_slots) {
 }
 }  // namespace
 
+// Tile buffers per CTA: double buffering (twice the tile memory, two CTAs per SM) where the
+// grid still fits one wave at that occupancy, or where a CTA walks three tiles or more (a long
+// loop gains more from overlapping its own gathers than from a single wave); a CTA of two
+// tiles in a larger grid relies on its co-resident CTAs to hide its gathers.
+static int draft_stages(const DraftPlan& plan, long units) {
+  return (plan.rows_per_split > kDRows && units * plan.n_split <= 2L * current_sm_count()) ||
+                 plan.rows_per_split > 2 * kDRows
+             ? 2
+             : 1;
+}
+// Entries of the CTA's row table: its slice rounded up to whole tiles.
+static int draft_pos_slots(const DraftPlan& plan) { return (plan.rows_per_split + kDRows - 1) / kDRows * kDRows; }
+
 // The kernel instance whose n8 query tiles hold a group of g query heads (g <= 16: one
 // tile up to 8, two beyond).
 int draft_group_instance(int g) { return g <= 1 ? 1 : g <= 2 ? 2 : g <= 4 ? 4 : g <= 8 ? 8 : 16; }
@@ -282,7 +295,7 @@ bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
   const long entries = (long)budget + n_steps;
   // one tile per CTA up to a cluster of 8, but no more CTAs than one wave holds at the
   // occupancy the slice's stage count gives (three single-stage or two double-buffered
-  // CTAs per SM, see launch_draft): a second wave would repeat the pass's whole latency chain
+  // CTAs per SM, draft_stages): a second wave would repeat the pass's whole latency chain
   const long units = (long)s.batch * s.h_kv;
   const long sms = current_sm_count();
   int n_split = (int)std::min<long>((entries + kDRows - 1) / kDRows, kDMaxCluster);
@@ -292,9 +305,14 @@ bool draft_plan(const bd_shape& s, int budget, int n_steps, DraftPlan* plan) {
     if (ctas <= (dbuf ? 2 : 3) * sms) break;
   }
   n_split = std::max(n_split, 1);
-  plan->rows_per_split = (int)((entries + n_split - 1) / n_split);
+  const long rows_per_split = (entries + n_split - 1) / n_split;
+  if (rows_per_split > (1L << 24)) return false;
+  plan->rows_per_split = (int)rows_per_split;
   plan->n_split = n_split;
-  return true;
+  // the row table of a CTA's slice sits in shared memory beside its tiles
+  const int g_kernel = draft_group_instance(g);
+  return smem_bytes(s.head_dim, g_kernel, draft_stages(*plan, units), n_split, draft_pos_slots(*plan)) <=
+         227 * 1024;
 }
 
 size_t draft_partials_bytes(const bd_shape&, const DraftPlan&) { return 0; }   // merged in the cluster
@@ -323,15 +341,8 @@ cudaError_t launch_draft(const bd_shape& s, const DraftPlan& plan, const void* q
   p.t_cap = s.t_cap;
   p.n_split = plan.n_split;
   p.rows_per_split = plan.rows_per_split;
-  // double buffering (twice the tile memory, two CTAs per SM) where the grid still fits one
-  // wave at that occupancy, or where a CTA walks three tiles or more (a long loop gains more
-  // from overlapping its own gathers than from a single wave); a CTA of two tiles in a
-  // larger grid relies on its co-resident CTAs to hide its gathers
-  p.n_stage = (plan.rows_per_split > kDRows && (long)units * plan.n_split <= 2L * current_sm_count()) ||
-                      plan.rows_per_split > 2 * kDRows
-                  ? 2
-                  : 1;
-  p.pos_slots = (plan.rows_per_split + kDRows - 1) / kDRows * kDRows;
+  p.n_stage = draft_stages(plan, units);
+  p.pos_slots = draft_pos_slots(plan);
   p.flags = flags;
   p.scale_log2 = kLog2e / sqrtf((float)s.head_dim);
   const int g = s.h_q / s.h_kv;

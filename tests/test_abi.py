@@ -93,6 +93,15 @@ def test_draft_validation(lib):
     assert draft(lib, shape(), flags=6) == INVALID                    # unknown flag bits
 
 
+def test_draft_view_beyond_shared_memory_is_unsupported(lib):
+    """The row table of a CTA's slice lives in shared memory: a view of a million entries
+    cannot be planned (size 0, BD_ERR_UNSUPPORTED), a 4K view can."""
+    s = shape(t_ctx=2_000_000, t_cap=2_000_010)
+    assert lib.bd_workspace_size(ctypes.byref(s), binding.BD_OP_DRAFT, 1_000_000, 1) == 0
+    assert lib.bd_workspace_size(ctypes.byref(s), binding.BD_OP_DRAFT, 4096, 1) > 0
+    assert draft(lib, s, budget=1_000_000) == UNSUPPORTED
+
+
 def test_select_validation(lib):
     assert select(lib, shape(), window=0) == INVALID
     assert select(lib, shape(), window=101) == INVALID                # window > t_ctx
