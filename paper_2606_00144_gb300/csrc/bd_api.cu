@@ -185,7 +185,7 @@ int bd_select_budget(const bd_shape* shape, const void* k_cache, const void* q_w
   BD_TRY(check_tensor(count_out, 4));
   if (window < 1 || window > s.t_ctx || budget < 1 || n_sink < 0 || n_recent < 0 || chunk < 1)
     return BD_ERR_INVALID_ARG;
-  if (budget < s.t_ctx && n_sink + n_recent > budget) return BD_ERR_INVALID_ARG;
+  if (budget < s.t_ctx && (long long)n_sink + n_recent > budget) return BD_ERR_INVALID_ARG;
   if (flags & ~BD_SELECT_WINDOW_READY) return BD_ERR_INVALID_ARG;
   if ((s.h_q / s.h_kv) * window > 256) return BD_ERR_UNSUPPORTED;
   SelectPlan sp;
@@ -322,7 +322,7 @@ int bd_advance(const bd_shape* shape, int window, int n_q, const int32_t* n_acce
                int idx_capacity, int32_t* advance_out, void* stream) {
   BD_TRY(check_shape(shape));
   const bd_shape& s = *shape;
-  if (window < 1 || window > s.t_ctx || n_q < 1 || s.t_ctx + n_q > s.t_cap) return BD_ERR_INVALID_ARG;
+  if (window < 1 || window > s.t_ctx || n_q < 1 || (long long)s.t_ctx + n_q > s.t_cap) return BD_ERR_INVALID_ARG;
   if ((verify_lse == nullptr) != (window_lse == nullptr)) return BD_ERR_INVALID_ARG;
   if ((idx == nullptr) != (count == nullptr)) return BD_ERR_INVALID_ARG;
   if (idx && idx_capacity < 1) return BD_ERR_INVALID_ARG;
@@ -348,7 +348,7 @@ int bd_write_block_rows(const bd_shape* shape, int n_rows, const void* k_rows, c
                         void* v_cache, void* stream) {
   BD_TRY(check_shape(shape));
   const bd_shape& s = *shape;
-  if (n_rows < 1 || s.t_ctx + n_rows > s.t_cap) return BD_ERR_INVALID_ARG;
+  if (n_rows < 1 || (long long)s.t_ctx + n_rows > s.t_cap) return BD_ERR_INVALID_ARG;
   BD_TRY(check_tensor(k_rows, 16));
   BD_TRY(check_tensor(v_rows, 16));
   BD_TRY(check_tensor(k_cache, 16));

@@ -77,6 +77,7 @@ def test_verify_validation(lib):
     assert verify(lib, shape(), o=A + 2) == MISALIGNED
     assert verify(lib, shape(), n_q=0) == INVALID
     assert verify(lib, shape(), n_q=11) == INVALID                    # t_ctx + n_q > t_cap
+    assert verify(lib, shape(), n_q=2**31 - 1) == INVALID             # the sum does not wrap
     assert verify(lib, shape(), o=0, lse=0) == INVALID                # nothing to write
     assert verify(lib, shape(t_cap=400), n_q=193) == UNSUPPORTED      # 4 * 193 rows > 768 with V
     assert verify(lib, shape(t_cap=200), n_q=33, o=0) == UNSUPPORTED  # 4 * 33 rows > 128, lse only
@@ -87,6 +88,7 @@ def test_draft_validation(lib):
     assert draft(lib, shape(), cnt=A + 2) == MISALIGNED
     assert draft(lib, shape(), j=-1) == INVALID
     assert draft(lib, shape(), j=10) == INVALID                       # t_ctx + j >= t_cap
+    assert draft(lib, shape(), j=2**31 - 1) == INVALID                # the sum does not wrap
     assert draft(lib, shape(), budget=0) == INVALID
     assert draft(lib, shape(h_q=34, h_kv=2)) == UNSUPPORTED           # group of 17 > 16
     assert draft(lib, shape(h_q=18, h_kv=2)) != UNSUPPORTED           # group of 9: two query tiles
@@ -106,6 +108,7 @@ def test_select_validation(lib):
     assert select(lib, shape(), window=0) == INVALID
     assert select(lib, shape(), window=101) == INVALID                # window > t_ctx
     assert select(lib, shape(), budget=10, sink=4, recent=8) == INVALID   # sink + recent > budget
+    assert select(lib, shape(), budget=10, sink=2**31 - 1, recent=2**31 - 1) == INVALID   # no wrap
     assert select(lib, shape(), chunk=0) == INVALID
     assert select(lib, shape(), flags=2) == INVALID                   # unknown flag bits
     assert select(lib, shape(), sink=-1) == INVALID
@@ -170,6 +173,7 @@ def test_advance_validation(lib):
     assert adv(shape(), window=0) == INVALID
     assert adv(shape(), window=101) == INVALID                          # window > t_ctx
     assert adv(shape(), n_q=11) == INVALID                              # t_ctx + n_q > t_cap
+    assert adv(shape(), n_q=2**31 - 1) == INVALID                       # the sum does not wrap
     assert adv(shape(), lv=None) == INVALID                             # lse ring needs both sides
     assert adv(shape(), cnt=None) == INVALID                            # view needs idx and count
     assert adv(shape(), cap=0) == INVALID
@@ -183,6 +187,7 @@ def test_write_block_rows_validation(lib):
     f = lib.bd_write_block_rows
     assert f(ctypes.byref(shape()), 0, A, A, A, A, None) == INVALID
     assert f(ctypes.byref(shape()), 11, A, A, A, A, None) == INVALID      # t_ctx + n_rows > t_cap
+    assert f(ctypes.byref(shape()), 2**31 - 1, A, A, A, A, None) == INVALID   # the sum does not wrap
     assert f(ctypes.byref(shape()), 6, A + 8, A, A, A, None) == MISALIGNED
     assert f(ctypes.byref(shape()), 6, A, A, None, A, None) == INVALID
     assert f(ctypes.byref(shape(head_dim=96)), 6, A, A, A, A, None) == UNSUPPORTED
