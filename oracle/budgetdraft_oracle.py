@@ -36,6 +36,24 @@ Readings where the paper is silent:
   * query i of a verify block sits at position t_ctx + i and sees keys
     [0, t_ctx + i]; draft pass j sees the selected rows plus its own rows
     t_ctx .. t_ctx + j.
+
+Pins (tests/test_oracle.py, CPU; none of this module is "parity unpinned"):
+  * attention: hand-derived basis fixture, identical keys -> mean value, one-hot
+    values -> the probabilities, shift invariance, single and empty key sets;
+  * verify_attn: hand-derived causal fixture, torch fp64 SDPA with a causal block
+    mask, one query = decode over the prefix;
+  * draft_attn: torch fp64 SDPA over the gathered rows, full budget = full attention;
+  * window_lse / window_scores (and window_positions): scipy logsumexp, torch softmax,
+    scores summing to G * W, a hand-derived uniform fixture;
+  * select_from_scores / select_budget (and topk_lower_index): exhaustive subset
+    enumeration with integer and real scores and ties (token and chunk level), all
+    equal keys, monotonicity in a planted shift, carried LSE = recomputed LSE;
+  * boundary_score: a fixture whose last admitted and first excluded scores differ;
+  * combine: a hand-derived fixture, disjoint parts = union, all parts empty;
+  * spec_step: brute-force selection over torch-softmax scores and fp64 SDPA;
+  * greedy_argmax / accept_greedy: fixtures and brute force with ties, NaN, signed
+    zeros; batch_advance / advance_window / append_view: closed cases and the window
+    of the longer context; widen_bf16_bits: exact against torch's bf16 widening.
 """
 
 from __future__ import annotations
