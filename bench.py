@@ -18,7 +18,8 @@ launching stream inside the timed region.  The step is captured in a CUDA graph;
 import os
 import sys
 
-if "OMP_NUM_THREADS" not in os.environ:           # the CPU baseline (numpy) uses every host core
+if "OMP_NUM_THREADS" not in os.environ:   # host-side numpy here may use every core (the oracle's
+                                          # worker processes run one BLAS thread each: OraclePool)
     _n = str(len(os.sched_getaffinity(0)))
     for _v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
         os.environ.setdefault(_v, _n)
@@ -775,7 +776,8 @@ def cpu_baseline(wl, budget, n_recent, sel_mode, budget_s=12.0, pool=None):
     return {"value": round(step_b / secs / 1e9, 4), "unit": "GB/s", "cores": pool.n, "kind": "oracle",
             "us_per_step": round(1e6 * secs, 1),
             "sample": f"{passes} whole steps of one layer ({wl.batch * wl.h_kv} (sequence, KV head) units, each the "
-                      f"selection with the carried window LSE, {wl.gamma} draft passes and the verify block), the "
+                      f"selection with {'the carried' if sel_mode == 'carry' else 'its own'} window LSE, "
+                      f"{wl.gamma} draft passes and the verify block), the "
                       f"units spread over {pool.n} single-threaded processes; numpy fp64"}
 
 
