@@ -371,7 +371,7 @@ def test_combine_merges_disjoint_draft_views():
 def test_tied_scores_take_lowest_positions(planted):
     """Middle keys set to zero have exactly equal scores: all of them (planted = 0: min = max)
     or all but every planted-th key, with the boundary falling among the ties in a bin too
-    crowded to rank, so the exact radix select runs (split over a cluster of CTAs)."""
+    crowded to rank, so the exact radix select runs."""
     wl = W.tiny_workload(batch=1, h_q=8, h_kv=2, head_dim=128, t_ctx=6000, budget=300, n_sink=4, n_recent=32,
                          window=32, gamma=1)
     inp = W.make_layer(wl, 0, "cuda")
